@@ -1,0 +1,318 @@
+"""Pins for the CPU oracle, each against something other than the oracle:
+brute force with a different algorithm, closed forms from App. B, invariants
+the paper states, and library routines.  CPU only."""
+import json
+import os
+
+import numpy as np
+import pytest
+import torch
+
+import brute
+import oracle
+from eqb_workloads import even_offsets, ragged_offsets
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def rand_bits(rng, T, E, scale=1.0, ties=False):
+    if ties:
+        # integer-valued logits in a tiny range: many exact ties in s = z + 0
+        v = rng.integers(-3, 4, size=(T, E)).astype(np.float32) * 0.5
+    else:
+        v = (rng.standard_normal((T, E)) * scale).astype(np.float32)
+    return brute.bf16_bits_from_f32(v)
+
+
+# ---------------------------------------------------------------- encodings
+
+def test_bf16_rounding_matches_torch():
+    rng = np.random.default_rng(1)
+    x = np.concatenate([
+        rng.standard_normal(20000).astype(np.float32),
+        (rng.standard_normal(2000) * 1e-39).astype(np.float32),   # fp32 subnormals
+        np.array([0.0, -0.0, 1.0 + 2**-8, 1.0 + 3 * 2**-8, -(1.0 + 2**-8), 2**-133,
+                  2**-134, 2**-135, -(2**-134), 3.0e38, -3.0e38, 1.7e38], dtype=np.float32),
+        rng.integers(0, 2**32, 20000, dtype=np.uint64).astype(np.uint32).view(np.float32),
+    ])
+    x = x[np.isfinite(x)]
+    want = brute.bf16_bits_from_f32(x)
+    got = np.array([oracle.f32_to_bf16_bits(v) for v in x], dtype=np.uint16)
+    # torch may saturate differently only for values that round past bf16 max
+    fin = np.isfinite(brute.f32_from_bf16_bits(want))
+    assert np.array_equal(got[fin], want[fin])
+
+
+def test_kappa_is_order_preserving_and_invertible():
+    allb = np.arange(65536, dtype=np.uint32).astype(np.uint16)
+    vals = brute.f32_from_bf16_bits(allb)
+    fin = np.isfinite(vals)
+    keys = np.array([oracle.kappa(int(x)) for x in allb])
+    assert len(set(keys.tolist())) == 65536
+    assert all(oracle.kappa_inv(int(k)) == int(x) for k, x in zip(keys, allb))
+    fk, fv = keys[fin], vals[fin]
+    order = np.argsort(fk, kind="stable")
+    sv = fv[order]
+    assert np.all(sv[1:] >= sv[:-1])  # keys sort values ascending (-0 just below +0)
+
+
+# ---------------------------------------------------------------- routing
+
+@pytest.mark.parametrize("E", [2, 3, 8])
+@pytest.mark.parametrize("ties", [False, True])
+def test_route_matches_repeated_extraction(E, ties):
+    rng = np.random.default_rng(10 + E + 100 * ties)
+    T = 40
+    z = rand_bits(rng, T, E, ties=ties)
+    b = np.zeros(E, np.float32) if ties else (rng.standard_normal(E) * 0.3).astype(np.float32)
+    for K in range(1, E):
+        idx, tau, loads = oracle.route(z, b, K)
+        for t in range(T):
+            want_idx, want_tau = brute.topk_by_extraction(brute.scores(z[t], b), K)
+            assert list(idx[t]) == want_idx
+            assert np.float32(tau[t]).tobytes() == np.float32(want_tau).tobytes()
+
+
+def test_cutoff_is_lower_endpoint_of_threshold_identity():
+    rng = np.random.default_rng(3)
+    E = 8
+    z = rand_bits(rng, 24, E)
+    b = (rng.standard_normal(E) * 0.5).astype(np.float32)
+    for K in (1, 2, 5, 7):
+        _, tau, _ = oracle.route(z, b, K)
+        for t in range(24):
+            s = brute.scores(z[t], b)
+            alpha, value = brute.cutoff_by_threshold_identity(s, K)
+            assert float(tau[t]) == float(alpha)
+            topk_sum = sum(sorted(s, reverse=True)[:K])
+            assert abs(float(value) - float(topk_sum)) < 1e-5
+
+
+def test_loads_sum_to_K_times_tokens():
+    rng = np.random.default_rng(4)
+    T, E = 999, 16
+    z = rand_bits(rng, T, E)
+    b = (rng.standard_normal(E) * 0.2).astype(np.float32)
+    for off in (even_offsets(T, 7), ragged_offsets(T, 9, 5)):
+        for K in (1, 4, 15):
+            idx, _, loads = oracle.route(z, b, K, off)
+            n = np.diff(off)
+            assert np.array_equal(loads.sum(1), K * n)
+            assert loads.sum() == K * T
+            # each token's list is K distinct experts
+            assert all(len(set(r)) == K for r in idx)
+            # loads are exactly the per-microbatch counts of the index lists
+            for l in range(len(n)):
+                cnt = np.bincount(idx[off[l]:off[l + 1]].ravel(), minlength=E)
+                assert np.array_equal(cnt, loads[l])
+
+
+# ---------------------------------------------------------------- quantile
+
+def test_quantile_is_smallest_minimiser_of_app_b_objective():
+    rng = np.random.default_rng(6)
+    for ties in (False, True):
+        T, E = 30, 6
+        z = rand_bits(rng, T, E, ties=ties)
+        b = np.zeros(E, np.float32)
+        for K in (1, 2, 5):
+            _, tau, _ = oracle.route(z, b, K)
+            r = oracle.target_rank(T, E, K)
+            q = oracle.quantile(z, tau, r)
+            for e in range(E):
+                m = brute.f32_from_bf16_bits(oracle.margins(z, tau, e))
+                want = brute.quantile_by_objective(m, r)
+                assert float(brute.f32_from_bf16_bits(q[e:e + 1])[0]) == float(want)
+
+
+def test_quantile_counting_invariant():
+    rng = np.random.default_rng(7)
+    T, E, K = 5000, 32, 4
+    z = rand_bits(rng, T, E)
+    b = (rng.standard_normal(E) * 0.3).astype(np.float32)
+    _, tau, _ = oracle.route(z, b, K)
+    r = oracle.target_rank(T, E, K)
+    q = brute.f32_from_bf16_bits(oracle.quantile(z, tau, r))
+    for e in range(E):
+        m = brute.f32_from_bf16_bits(oracle.margins(z, tau, e))
+        assert np.sum(m < q[e]) < r <= np.sum(m <= q[e])
+
+
+@pytest.mark.parametrize("parts", [[1], [3, 5, 8], [64]])
+def test_radix_selection_equals_full_sort(parts):
+    """Algorithm 1 run literally (brute, Python) over any partition of the
+    tokens into ranks returns the full-sort quantile, and so do the oracle's
+    own step functions; the summed per-rank counts equal the whole-batch
+    counts (P:111 partition invariance)."""
+    rng = np.random.default_rng(8)
+    T, E, K = 600, 8, 2
+    z = rand_bits(rng, T, E, scale=0.7)
+    b = (rng.standard_normal(E) * 0.2).astype(np.float32)
+    _, tau, _ = oracle.route(z, b, K)
+    r = oracle.target_rank(T, E, K)
+    q_sort = oracle.quantile(z, tau, r)
+    H_all = oracle.hist_hi(z, tau)
+    u, rho = oracle.select_hi(H_all, r)
+    q_steps = oracle.select_lo(oracle.hist_lo(z, tau, u), u, rho)
+    assert np.array_equal(q_steps, q_sort)
+    for P in parts:
+        perm = rng.permutation(T)
+        cuts = np.sort(rng.choice(np.arange(1, T), size=P - 1, replace=False)) if P > 1 else []
+        bounds = np.concatenate([[0], cuts, [T]]).astype(int)
+        zp, taup = z[perm], tau[perm]
+        H_sum = sum(oracle.hist_hi(zp, taup, bounds[p], bounds[p + 1]) for p in range(P))
+        assert np.array_equal(H_sum, H_all)
+        L_sum = sum(oracle.hist_lo(zp, taup, u, bounds[p], bounds[p + 1]) for p in range(P))
+        assert np.array_equal(oracle.select_lo(L_sum, u, rho), q_sort)
+        for e in range(E):
+            m = oracle.margins(zp, taup, e)
+            ranks = [m[bounds[p]:bounds[p + 1]] for p in range(P)]
+            assert brute.radix_select_alg1(ranks, r) == int(q_sort[e])
+
+
+def test_token_permutation_changes_no_quantile_or_global_load():
+    rng = np.random.default_rng(9)
+    T, E, K = 1000, 16, 3
+    z = rand_bits(rng, T, E)
+    b = (rng.standard_normal(E) * 0.2).astype(np.float32)
+    a = oracle.eqb_step(z, b, K)
+    perm = rng.permutation(T)
+    p = oracle.eqb_step(z[perm], b, K)
+    assert np.array_equal(a["qhat"], p["qhat"])
+    assert np.array_equal(a["loads"].sum(0), p["loads"].sum(0))
+    assert np.array_equal(a["tau"][perm], p["tau"])
+
+
+# ---------------------------------------------------------------- closed forms
+
+def cyclic_logits(T, E, K):
+    """App. B: enumerate the TK slots cyclically over the E experts;
+    token t owns slots tK .. tK+K-1.  z = 1 on owned experts, else 0."""
+    z = np.zeros((T, E), np.float32)
+    for t in range(T):
+        for j in range(K):
+            z[t, (t * K + j) % E] = 1.0
+    return brute.bf16_bits_from_f32(z)
+
+
+def test_cyclic_balanced_assignment_golden():
+    with open(os.path.join(GOLDEN, "cyclic_balanced.json")) as f:
+        cases = json.load(f)["cases"]
+    for c in cases:
+        T, E, K, M = c["T"], c["E"], c["K"], c["M"]
+        z = cyclic_logits(T, E, K)
+        b = np.zeros(E, np.float32)
+        off = even_offsets(T, M)
+        st = oracle.eqb_step(z, b, K, off)
+        assert st["r"] == c["r"]
+        assert np.all(st["loads"].sum(0) == c["r"])
+        assert np.all(st["loads"] == c["load_per_microbatch"])
+        assert np.all(st["tau"] == c["tau"])
+        assert np.all(brute.f32_from_bf16_bits(st["qhat"]) == c["qhat"])
+        assert np.all(st["b_next"] == c["b_next"])
+        g = np.random.default_rng(2).standard_normal((T, E)).astype(np.float32)
+        g_out, a = oracle.lei(g, st["loads"], off, K, eta=0.5, c=1.0)
+        assert np.all(a == c["lei_coefficient"])
+        assert np.array_equal(g_out, g)
+
+
+def test_constant_columns_closed_form():
+    """z_{t,e} = c_e for all t, b = 0: every token has the same top-K and
+    cutoff tau = c_(K+1); every margin of expert e equals bf16(tau - c_e), so
+    b_hat_e = that value; loads are n_l on the top-K experts and 0 elsewhere,
+    giving rho = E/K - 1 or -1 and the LEI coefficient of Eq. (norm)."""
+    E, K, T = 8, 3, 120
+    cvals = np.array([0.5, -1.25, 2.0, 0.75, -0.5, 1.5, 0.25, -2.0], np.float32)
+    z = np.tile(brute.bf16_bits_from_f32(cvals), (T, 1))
+    b = np.zeros(E, np.float32)
+    off = np.array([0, 50, 120], np.int64)
+    st = oracle.eqb_step(z, b, K, off)
+    order = sorted(range(E), key=lambda e: (-cvals[e], e))
+    assert all(list(r) == order[:K] for r in st["idx"])
+    tau = cvals[order[K]]
+    assert np.all(st["tau"] == tau)
+    want_q = brute.bf16_bits_from_f32(np.float32(tau) - cvals)
+    want_q[want_q == 0x8000] = 0
+    assert np.array_equal(st["qhat"], want_q)
+    eta, c = 0.01, 1.5
+    _, a = oracle.lei(None, st["loads"], off, K, eta, c)
+    rho = np.where(np.isin(np.arange(E), order[:K]), E / K - 1.0, -1.0)
+    xi = np.abs(rho).max() / c
+    eta_f = float(np.float32(eta))  # the interface takes eta and c as fp32
+    xi = np.abs(rho).max() / float(np.float32(c))
+    assert np.allclose(a, eta_f * np.tanh(xi) / xi * rho[None, :], rtol=1e-13, atol=0)
+
+
+# ---------------------------------------------------------------- LEI
+
+def test_lei_invariants():
+    rng = np.random.default_rng(12)
+    T, E, K = 3000, 32, 4
+    z = rand_bits(rng, T, E)
+    b = (rng.standard_normal(E) * 0.3).astype(np.float32)
+    off = ragged_offsets(T, 6, 3)
+    _, _, loads = oracle.route(z, b, K, off)
+    g = (rng.standard_normal((T, E)) * 0.1).astype(np.float32)
+    n = np.diff(off)
+    for c in (0.5, 1.0, 4.0, 0.0):
+        eta = float(np.float32(0.7))  # the interface takes eta as fp32
+        g_out, a = oracle.lei(g, loads, off, K, eta, c)
+        for l in range(len(n)):
+            if n[l] == 0:
+                assert np.all(a[l] == 0)
+                continue
+            fbar = K * n[l] / E
+            rho = loads[l] / fbar - 1.0
+            assert abs(rho.sum()) < 1e-9                                  # zero-centred
+            assert np.all(np.sign(a[l]) == np.sign(loads[l] - fbar))      # direction
+            rt = a[l] / eta
+            if c > 0:
+                xi = np.abs(rho).max() / c
+                assert np.isclose(np.abs(rt).max(), c * np.tanh(xi), rtol=1e-12)
+                assert np.abs(rt).max() < c                               # bounded (Eq. norm)
+                assert np.allclose(rt / rho, np.tanh(xi) / xi, rtol=1e-12)  # one shared scale
+            else:
+                assert np.allclose(rt, rho, rtol=1e-12)                   # unnormalised Eq. (LEI)
+            seg = slice(off[l], off[l + 1])
+            want = (g[seg].astype(np.float64) + a[l][None, :]).astype(np.float32)
+            assert np.array_equal(g_out[seg], want)
+    g0, a0 = oracle.lei(g, loads, off, K, 0.0, 1.0)
+    assert np.array_equal(g0, g) and np.all(a0 == 0)
+
+
+def test_lei_scale_limit_at_zero():
+    """tanh(xi)/xi -> 1 as xi -> 0: a perfectly balanced microbatch has a = 0,
+    and a tiny imbalance with large c gives a ~= eta * rho."""
+    E, K = 4, 1
+    off = np.array([0, 4000], np.int64)
+    loads = np.array([[1000, 1000, 1000, 1000]], np.int32)
+    _, a = oracle.lei(None, loads, off, K, 2.0, 1.0)
+    assert np.all(a == 0)
+    loads = np.array([[1001, 999, 1000, 1000]], np.int32)
+    _, a = oracle.lei(None, loads, off, K, 2.0, 1e6)
+    rho = loads[0] / 1000.0 - 1.0
+    assert np.allclose(a[0], 2.0 * rho, rtol=1e-9)
+
+
+# ---------------------------------------------------------------- bias update
+
+def test_bias_update_centering():
+    rng = np.random.default_rng(13)
+    q = brute.bf16_bits_from_f32((rng.standard_normal(256) * 2).astype(np.float32))
+    bn = oracle.bias_update(q)
+    qv = brute.f32_from_bf16_bits(q).astype(np.float64)
+    mean = qv.sum() / 256  # exact here: all partial sums fit in fp64
+    assert np.array_equal(bn, (qv - mean).astype(np.float32))
+    assert abs(bn.astype(np.float64).sum()) < 256 * 2**-22
+    # a common shift of b_hat leaves the update unchanged when exact
+    shifted = brute.bf16_bits_from_f32(brute.f32_from_bf16_bits(q).astype(np.float32))
+    assert np.array_equal(oracle.bias_update(shifted), bn)
+
+
+def test_target_rank():
+    assert oracle.target_rank(4096, 8, 2) == 1024
+    assert oracle.target_rank(65536, 64, 8) == 8192
+    assert oracle.target_rank(524288, 128, 8) == 32768
+    assert oracle.target_rank(2097152, 256, 8) == 65536
+    assert oracle.target_rank(1048576, 128, 8) == 65536
+    assert oracle.target_rank(10, 8, 3) == 4  # ceil(30/8)
