@@ -1,0 +1,159 @@
+/*
+ * eqb.h -- C ABI of libeqb.so: the per-layer MoE routing-balance path of
+ * Exact Quantile Balancing (EQB) and Load-Error Injection (LEI),
+ * arXiv 2609.28053, on one NVIDIA GB300 (sm_103a).
+ *
+ * Notation follows the paper: T tokens, E routed experts, K experts per
+ * token, router logits z[T,E], expert bias b[E], cutoff tau_t = the (K+1)st
+ * largest entry of z_t + b, expert loads f_e, target rank r = TK/E.
+ *
+ * Conventions shared by every call
+ * --------------------------------
+ *  - Pointers named as device buffers are CUDA device (or managed) pointers
+ *    that the caller allocates and owns.  Unless a function says otherwise,
+ *    the library allocates no device memory and keeps no state between calls.
+ *  - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *    stream).  Every call only enqueues work on it and returns without
+ *    synchronising; results are valid once the stream has reached them.
+ *  - Row-major layouts with the expert index fastest: z[t*E + e].
+ *  - bf16 values travel as their raw 16-bit patterns (eqb_bf16).
+ *  - Outputs documented as "+=" are accumulated into; the caller zeroes them
+ *    first.  This is what lets token partitions (the data-parallel ranks of
+ *    Algorithm 1, here slices of one batch) be summed in device memory, and
+ *    lets a multi-GPU caller insert its own all-reduce between passes.
+ *  - Return value: an eqb_status.  Arguments are validated on the host
+ *    before anything is launched; an invalid call launches nothing.
+ *    EQB_ERR_CUDA reports a launch failure (cudaGetLastError after launch).
+ *  - Errors found by the device (non-finite data, an unreachable rank) are
+ *    written to the optional device word `err_flag` (int32, nullable) as the
+ *    eqb_status code; the caller zeroes it before the call and reads it after
+ *    synchronising.  Outputs of a call that flagged an error are unspecified.
+ *  - Microbatches (the paper's local batches B_l, Sec. 2) are contiguous
+ *    token ranges given by device int64 offsets[M+1]: offsets[0] = 0,
+ *    offsets[M] = T, non-decreasing (empty microbatches are allowed).
+ *    The library reads them on the device; they are not checked on the host.
+ *  - Supported sizes: 1 <= K, K + 1 <= 32, K < E, E a multiple of 8 with
+ *    E <= 256, T < 2^31.  T = 0 is a valid no-op for the streaming calls.
+ *  - Device buffers of bf16 logits must be 16-byte aligned; fp32 gradient
+ *    buffers 16-byte aligned.  Misaligned pointers give EQB_ERR_INVALID_ARG.
+ */
+#ifndef EQB_H
+#define EQB_H
+
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+typedef uint16_t eqb_bf16; /* raw bf16 bit pattern */
+
+typedef enum eqb_status {
+  EQB_OK = 0,
+  EQB_ERR_INVALID_ARG = 1, /* host-side validation failed; nothing launched */
+  EQB_ERR_UNSUPPORTED = 2, /* valid by the paper, outside this build's sizes */
+  EQB_ERR_CUDA = 3,        /* a CUDA launch or runtime call failed */
+  EQB_ERR_NONFINITE = 4,   /* device flag: non-finite z, b or score, or a
+                              margin of magnitude >= 2^127 */
+  EQB_ERR_RANK = 5         /* device flag: a histogram holds fewer than r
+                              margins for some expert */
+} eqb_status;
+
+/* Human-readable name of a status code (static string). */
+const char *eqb_status_string(int status);
+
+/* Library version as MAJOR*10000 + MINOR*100 + PATCH. */
+int eqb_version(void);
+
+/* Target rank r = ceil(T*K / E) (Sec. 3: r = TK/E, assumed integral by the
+ * paper; rounded up otherwise, the inverse-CDF quantile).  Returns -1 for
+ * invalid arguments.  Host only. */
+int64_t eqb_target_rank(int64_t T, int32_t E, int32_t K);
+
+/* Routing and the coarse EQB pass.  Sec. 2 (Eq. 1 and the QB paragraph),
+ * Algorithm 1 step 1.
+ *
+ * For each token t: s_e = fp32(z_{t,e}) + b_e (fp32, round to nearest
+ * even); the top-K set of s (ties to the lower expert index), written to
+ * topk_idx[t, 0..K-1] in descending score order; tau[t] = the (K+1)st
+ * largest s (fp32).  loads[l, e] += number of tokens of microbatch l whose
+ * top-K set contains e.
+ *
+ * hist_hi (nullable): when given, also accumulates Algorithm 1's coarse
+ * histogram: for every (t, e), the margin m = bf16_rne(tau_t - fp32(z_{t,e}))
+ * is encoded by the order-preserving key kappa(m) (bf16 pattern x ->
+ * x & 0x8000 ? ~x : x | 0x8000, 16 bits) and hist_hi[e, kappa(m) >> 8] += 1.
+ *
+ *   z         device bf16 [T,E], 16-byte aligned          (in)
+ *   b         device fp32 [E]                              (in)
+ *   mb_offsets device int64 [M+1] (nullable iff loads is NULL)
+ *   topk_idx  device int32 [T,K]   (nullable)              (out)
+ *   tau       device fp32 [T]                              (out)
+ *   loads     device int32 [M,E] += (nullable)             (in/out)
+ *   hist_hi   device int32 [E,256] += (nullable)           (in/out)
+ *   err_flag  device int32 (nullable): EQB_ERR_NONFINITE for a non-finite
+ *             b_e or NaN score, or (with hist_hi) a non-finite margin.
+ */
+eqb_status eqb_route_topk(const eqb_bf16 *z, const float *b, int64_t T, int32_t E,
+                          int32_t K, const int64_t *mb_offsets, int32_t M,
+                          int32_t *topk_idx, float *tau, int32_t *loads,
+                          int32_t *hist_hi, int32_t *err_flag, void *stream);
+
+/* Coarse pass on its own (Algorithm 1 step 1): recomputes the margins from z
+ * and tau and accumulates hist_hi[e, kappa(m) >> 8] += 1 over T tokens.
+ * Margins of magnitude >= 2^127 or non-finite set EQB_ERR_NONFINITE. */
+eqb_status eqb_margin_hist_pass1(const eqb_bf16 *z, const float *tau, int64_t T,
+                                 int32_t E, int32_t *hist_hi, int32_t *err_flag,
+                                 void *stream);
+
+/* Fine pass (Algorithm 1 step 4; Sec. 3 "the second pass simply rescans
+ * local margins whose high byte matches the selected bin"): recomputes
+ * every margin from z and tau and, where kappa(m) >> 8 == u[e], accumulates
+ * hist_lo[e, kappa(m) & 0xff] += 1.  No margin array is materialised.
+ *   u        device uint8 [E] (from eqb_select_quantile pass 1)
+ *   hist_lo  device int32 [E,256] += */
+eqb_status eqb_margin_hist_pass2(const eqb_bf16 *z, const float *tau, int64_t T,
+                                 int32_t E, const uint8_t *u, int32_t *hist_lo,
+                                 void *stream);
+
+/* Selection on a summed histogram (Algorithm 1 steps 3, 5 and 6).
+ *   pass 1: reads hist = H [E,256]; writes u[e] = min{u : sum_{j<=u} H[e,j]
+ *           >= r} and rho[e] = r - sum_{j<u_e} H[e,j].  r is the global
+ *           target rank (eqb_target_rank of the whole batch).  Sets
+ *           EQB_ERR_NONFINITE if a margin landed in high byte 0x00 or 0xff
+ *           (magnitude >= 2^127 or non-finite) and EQB_ERR_RANK if H[e,:]
+ *           sums to less than r.
+ *   pass 2: reads hist = L [E,256], u and rho; writes v_e = min{v :
+ *           sum_{j<=v} L[e,j] >= rho_e} and q_hat[e] = kappa^{-1}((u_e << 8)
+ *           | v_e), the exact r-th smallest margin (a zero as +0).
+ *   q_hat is ignored in pass 1; r is ignored in pass 2. */
+eqb_status eqb_select_quantile(const int32_t *hist, int32_t E, int32_t pass,
+                               int64_t r, uint8_t *u, int32_t *rho, eqb_bf16 *q_hat,
+                               int32_t *err_flag, void *stream);
+
+/* Bias update of Eq. (2): b_next[e] = (float)((double)q_hat[e] - mean) with
+ * mean = (sum over e = 0..E-1 in ascending order, in fp64) / E.  The fixed
+ * order makes the result bit-reproducible.  b_next is used for routing in
+ * the next optimizer step. */
+eqb_status eqb_bias_update(const eqb_bf16 *q_hat, int32_t E, float *b_next,
+                           void *stream);
+
+/* Load-Error Injection, Sec. 4 Eq. (LEI) with the normalisation Eq. (norm).
+ * For each microbatch l with n_l tokens (empty ones are skipped):
+ *   rho_e = f_{l,e} / (K n_l / E) - 1;
+ *   c > 0:  xi = max_e |rho_e| / c,  sigma = tanh(xi) / xi (1 at xi = 0);
+ *   c <= 0: sigma = 1 (unnormalised LEI);
+ *   grad_s[t, e] += eta * sigma * rho_e for every t in the microbatch and
+ *   every expert e.  The coefficient is formed in fp64, rounded to fp32,
+ *   and added in fp32.
+ *   grad_s  device fp32 [T,E], 16-byte aligned, updated in place
+ *   loads   device int32 [M,E] (the local loads from eqb_route_topk) */
+eqb_status lei_inject_grad(float *grad_s, const int32_t *loads,
+                           const int64_t *mb_offsets, int32_t M, int64_t T,
+                           int32_t E, int32_t K, float eta, float c, void *stream);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* EQB_H */

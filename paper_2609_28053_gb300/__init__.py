@@ -1,0 +1,175 @@
+"""GB300-native EQB + LEI routing-balance path (arXiv 2609.28053).
+
+Thin Python binding over the C ABI of ``libeqb.so`` (include/eqb.h).  Each
+function has the C entry point's name, checks dtypes/devices/shapes, and
+passes raw device pointers plus the current CUDA stream; every step of the
+path runs in the library's CUDA kernels.  PyTorch provides device memory
+and streams only.
+
+The routing-balance step of one MoE layer, in the paper's order:
+
+    eqb_route_topk        Sec. 2: top-K of z + b, cutoff tau_t, loads f_e
+                          (+ Algorithm 1 step 1, the coarse histogram)
+    eqb_select_quantile   Algorithm 1 step 3 (pass 1): u_e, rho_e
+    eqb_margin_hist_pass2 Algorithm 1 step 4: fine histogram
+    eqb_select_quantile   Algorithm 1 steps 5-6 (pass 2): exact quantile
+    eqb_bias_update       Eq. (2): centred bias for the next step
+    lei_inject_grad       Sec. 4: Eq. (LEI) with Eq. (norm)
+"""
+from __future__ import annotations
+
+import ctypes
+
+import torch
+
+from ._lib import STATUS, EqbError, load
+
+__all__ = [
+    "EqbError", "STATUS", "load", "eqb_target_rank", "eqb_route_topk", "eqb_margin_hist_pass1",
+    "eqb_margin_hist_pass2", "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad",
+    "EqbWorkspace", "eqb_layer_forward",
+]
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream):
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _need(t, dtype, name, shape=None):
+    if t is None:
+        return
+    if not isinstance(t, torch.Tensor):
+        raise TypeError(f"{name} must be a torch.Tensor")
+    if t.dtype != dtype:
+        raise TypeError(f"{name} must be {dtype}, got {t.dtype}")
+    if not t.is_cuda:
+        raise ValueError(f"{name} must be a CUDA tensor")
+    if not t.is_contiguous():
+        raise ValueError(f"{name} must be contiguous")
+    if shape is not None and tuple(t.shape) != tuple(shape):
+        raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
+
+
+def _check(rc, what):
+    if rc != 0:
+        raise EqbError(rc, what)
+
+
+def eqb_target_rank(T: int, E: int, K: int) -> int:
+    return int(load().eqb_target_rank(T, E, K))
+
+
+def eqb_route_topk(z, b, K, mb_offsets=None, topk_idx=None, tau=None, loads=None, hist_hi=None,
+                   err_flag=None, stream=None):
+    """Top-K routing, cutoffs and loads (+ optional coarse histogram).
+    z bf16 [T,E]; b fp32 [E]; mb_offsets int64 [M+1]; outputs as in eqb.h.
+    loads and hist_hi are accumulated into.  Returns (topk_idx, tau)."""
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(b, torch.float32, "b", (E,))
+    if tau is None:
+        tau = torch.empty(T, dtype=torch.float32, device=z.device)
+    _need(tau, torch.float32, "tau", (T,))
+    _need(topk_idx, torch.int32, "topk_idx", (T, K))
+    M = 0
+    if mb_offsets is not None:
+        _need(mb_offsets, torch.int64, "mb_offsets")
+        M = mb_offsets.numel() - 1
+    _need(loads, torch.int32, "loads", (M, E) if loads is not None else None)
+    _need(hist_hi, torch.int32, "hist_hi", (E, 256))
+    _need(err_flag, torch.int32, "err_flag")
+    rc = load().eqb_route_topk(_p(z), _p(b), T, E, K, _p(mb_offsets), M, _p(topk_idx), _p(tau),
+                               _p(loads), _p(hist_hi), _p(err_flag), _stream(stream))
+    _check(rc, "eqb_route_topk")
+    return topk_idx, tau
+
+
+def eqb_margin_hist_pass1(z, tau, hist_hi, err_flag=None, stream=None):
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(tau, torch.float32, "tau", (T,))
+    _need(hist_hi, torch.int32, "hist_hi", (E, 256))
+    _need(err_flag, torch.int32, "err_flag")
+    _check(load().eqb_margin_hist_pass1(_p(z), _p(tau), T, E, _p(hist_hi), _p(err_flag),
+                                        _stream(stream)), "eqb_margin_hist_pass1")
+
+
+def eqb_margin_hist_pass2(z, tau, u, hist_lo, stream=None):
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(tau, torch.float32, "tau", (T,))
+    _need(u, torch.uint8, "u", (E,))
+    _need(hist_lo, torch.int32, "hist_lo", (E, 256))
+    _check(load().eqb_margin_hist_pass2(_p(z), _p(tau), T, E, _p(u), _p(hist_lo), _stream(stream)),
+           "eqb_margin_hist_pass2")
+
+
+def eqb_select_quantile(hist, pass_, r, u, rho, q_hat=None, err_flag=None, stream=None):
+    E = hist.shape[0]
+    _need(hist, torch.int32, "hist", (E, 256))
+    _need(u, torch.uint8, "u", (E,))
+    _need(rho, torch.int32, "rho", (E,))
+    _need(q_hat, torch.bfloat16, "q_hat", (E,))
+    _need(err_flag, torch.int32, "err_flag")
+    _check(load().eqb_select_quantile(_p(hist), E, int(pass_), int(r), _p(u), _p(rho), _p(q_hat),
+                                      _p(err_flag), _stream(stream)), "eqb_select_quantile")
+
+
+def eqb_bias_update(q_hat, b_next, stream=None):
+    E = q_hat.shape[0]
+    _need(q_hat, torch.bfloat16, "q_hat", (E,))
+    _need(b_next, torch.float32, "b_next", (E,))
+    _check(load().eqb_bias_update(_p(q_hat), E, _p(b_next), _stream(stream)), "eqb_bias_update")
+
+
+def lei_inject_grad(grad_s, loads, mb_offsets, K, eta, c, stream=None):
+    T, E = grad_s.shape
+    _need(grad_s, torch.float32, "grad_s")
+    _need(mb_offsets, torch.int64, "mb_offsets")
+    M = mb_offsets.numel() - 1
+    _need(loads, torch.int32, "loads", (M, E))
+    _check(load().lei_inject_grad(_p(grad_s), _p(loads), _p(mb_offsets), M, T, E, K, float(eta),
+                                  float(c), _stream(stream)), "lei_inject_grad")
+
+
+class EqbWorkspace:
+    """Device buffers of one layer's EQB statistic: the two [E,256] int32
+    histograms, u, rho, q_hat and the error word.  Allocated once by the
+    caller (through torch), reused every step."""
+
+    def __init__(self, E: int, device="cuda"):
+        self.E = E
+        self.hist_hi = torch.zeros((E, 256), dtype=torch.int32, device=device)
+        self.hist_lo = torch.zeros((E, 256), dtype=torch.int32, device=device)
+        self.u = torch.zeros(E, dtype=torch.uint8, device=device)
+        self.rho = torch.zeros(E, dtype=torch.int32, device=device)
+        self.q_hat = torch.zeros(E, dtype=torch.bfloat16, device=device)
+        self.err = torch.zeros(1, dtype=torch.int32, device=device)
+
+    def zero_(self):
+        self.hist_hi.zero_()
+        self.hist_lo.zero_()
+        self.err.zero_()
+
+
+def eqb_layer_forward(z, b, K, mb_offsets, ws: EqbWorkspace, topk_idx, tau, loads, b_next,
+                      r=None, stream=None):
+    """One layer's forward routing-balance statistic, in the paper's order:
+    routing + coarse pass, select 1, fine pass, select 2, bias update.
+    `loads` must be zeroed by the caller (it is accumulated into); the
+    workspace histograms are zeroed here.  All steps run on `stream`."""
+    T, E = z.shape
+    if r is None:
+        r = eqb_target_rank(T, E, K)
+    ws.zero_()
+    eqb_route_topk(z, b, K, mb_offsets, topk_idx, tau, loads, ws.hist_hi, ws.err, stream)
+    eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream)
+    eqb_margin_hist_pass2(z, tau, ws.u, ws.hist_lo, stream)
+    eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err, stream)
+    eqb_bias_update(ws.q_hat, b_next, stream)

@@ -1,0 +1,80 @@
+// eqb_device.cuh -- device helpers shared by the EQB / LEI kernels.
+//
+// bf16 values are handled as raw 16-bit patterns packed two per 32-bit
+// word (lower half = lower expert index).  All fp32 arithmetic is IEEE
+// round-to-nearest-even without flush-to-zero (the library is built without
+// fast-math and with -fmad=false), so scores and margins are reproducible
+// bit for bit.
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "eqb_internal.h"
+
+namespace eqb {
+
+constexpr unsigned kFull = 0xffffffffu;
+
+// bf16 in the low / high half of a packed word -> fp32 (exact).
+__device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
+__device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }
+__device__ __forceinline__ float bf16_bits_to_f32(uint32_t x16) { return __uint_as_float(x16 << 16); }
+
+// Two fp32 values -> packed bf16x2, round to nearest even (lo -> low half).
+__device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
+  uint32_t r;
+  asm("cvt.rn.bf16x2.f32 %0, %1, %2;" : "=r"(r) : "f"(hi), "f"(lo));
+  return r;
+}
+
+// fp32 max that propagates NaN (used where a NaN must stay visible).
+__device__ __forceinline__ float fmax_nan(float a, float b) {
+  float r;
+  asm("max.NaN.f32 %0, %1, %2;" : "=f"(r) : "f"(a), "f"(b));
+  return r;
+}
+
+// Order-preserving 16-bit key of a bf16 pattern (Algorithm 1's kappa):
+// negative patterns are complemented, non-negative ones get the sign bit.
+__device__ __forceinline__ uint32_t kappa16(uint32_t x16) {
+  return (x16 & 0x8000u) ? (~x16 & 0xffffu) : (x16 | 0x8000u);
+}
+
+__device__ __forceinline__ uint32_t kappa16_inv(uint32_t k16) {
+  return (k16 & 0x8000u) ? (k16 & 0x7fffu) : (~k16 & 0xffffu);
+}
+
+// 16-byte shared-memory load.
+__device__ __forceinline__ uint4 lds128(const void* p) { return *reinterpret_cast<const uint4*>(p); }
+
+// Ampere-style asynchronous 16-byte global->shared copy (L2 only).  With
+// src_bytes = 0 nothing is read and the destination is zero-filled.
+__device__ __forceinline__ void cp_async16(void* smem_dst, const void* gmem_src, int src_bytes) {
+  uint32_t d = static_cast<uint32_t>(__cvta_generic_to_shared(smem_dst));
+  asm volatile("cp.async.cg.shared.global [%0], [%1], 16, %2;\n" ::"r"(d), "l"(gmem_src),
+               "r"(src_bytes)
+               : "memory");
+}
+__device__ __forceinline__ void cp_async_commit() { asm volatile("cp.async.commit_group;\n" ::: "memory"); }
+template <int N>
+__device__ __forceinline__ void cp_async_wait() {
+  asm volatile("cp.async.wait_group %0;\n" ::"n"(N) : "memory");
+}
+
+// Microbatch of token t: the largest l with off[l] <= t (empty microbatches
+// are skipped automatically).  Requires 0 <= t < off[M].
+__device__ __forceinline__ int microbatch_of(const int64_t* __restrict__ off, int M, int64_t t) {
+  int lo = 0, hi = M - 1;
+  while (lo < hi) {
+    int mid = (lo + hi + 1) >> 1;
+    if (__ldg(off + mid) <= t) lo = mid; else hi = mid - 1;
+  }
+  return lo;
+}
+
+__device__ __forceinline__ void raise_flag(int32_t* err, int code) {
+  if (err) atomicCAS(err, 0, code);
+}
+
+}  // namespace eqb

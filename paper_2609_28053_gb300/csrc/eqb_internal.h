@@ -1,0 +1,68 @@
+// eqb_internal.h -- launch-side declarations shared by the .cu files of
+// libeqb.so (not part of the public ABI; see include/eqb.h for that).
+#pragma once
+
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+namespace eqb {
+
+// Status codes mirrored from eqb.h for device code.
+enum : int {
+  kOk = 0,
+  kErrInvalidArg = 1,
+  kErrUnsupported = 2,
+  kErrCuda = 3,
+  kErrNonfinite = 4,
+  kErrRank = 5,
+};
+
+struct DeviceInfo {
+  int sm_count;
+  int max_smem_optin;  // bytes of dynamic shared memory a block may opt into
+};
+
+// Cached per-device attributes (queried once per device).
+int device_info(DeviceInfo* out);
+
+struct RouteArgs {
+  const uint16_t* z;
+  const float* b;
+  int64_t T;
+  int E, K;
+  const int64_t* off;
+  int M;
+  int32_t* idx;
+  float* tau;
+  int32_t* loads;
+  int32_t* err;
+};
+
+struct HistArgs {
+  const uint16_t* z;
+  const float* tau;
+  int64_t T;
+  int E;
+  const uint8_t* u;  // pass 2 only
+  int32_t* hist;
+  int32_t* err;
+};
+
+struct LeiArgs {
+  float* g;
+  const int32_t* loads;
+  const int64_t* off;
+  int M;
+  int64_t T;
+  int E, K;
+  float eta, c;
+};
+
+int launch_route(const RouteArgs& a, cudaStream_t s);
+int launch_hist(const HistArgs& a, int pass, cudaStream_t s);
+int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, int32_t* rho,
+                  uint16_t* q_hat, int32_t* err, cudaStream_t s);
+int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t s);
+int launch_lei(const LeiArgs& a, cudaStream_t s);
+
+}  // namespace eqb

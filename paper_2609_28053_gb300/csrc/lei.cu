@@ -1,0 +1,121 @@
+// lei.cu -- Load-Error Injection (arXiv 2609.28053, Sec. 4, Eq. (LEI) and
+// Eq. (norm)).
+//
+// For microbatch l with n_l tokens and loads f_{l,e}:
+//   rho_e = f_{l,e} / (K n_l / E) - 1,
+//   sigma = tanh(xi) / xi with xi = max_e |rho_e| / c   (c > 0; 1 at xi = 0),
+//   sigma = 1                                            (c <= 0, unnormalised),
+//   grad_s[t, e] += eta * sigma * rho_e   for every t of the microbatch, every e.
+//
+// The path is a pure HBM stream (read and write grad_s once), so each CTA
+// takes a contiguous token range, computes the E coefficients of each
+// microbatch it meets (fp64, one thread per expert, a block max for xi) into
+// shared memory as fp32, and then streams its range with 16-byte loads and
+// stores using evict-first cache hints.
+#include "eqb_device.cuh"
+
+namespace eqb {
+
+namespace {
+
+constexpr int kLeiThreads = 256;
+constexpr int kLeiUnroll = 4;
+
+__global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tokens_per_cta) {
+  __shared__ __align__(16) float coef[256];
+  __shared__ double red[kLeiThreads / 32];
+  const int E = a.E, E4 = a.E >> 2;
+  const int64_t tb = (int64_t)blockIdx.x * tokens_per_cta;
+  const int64_t te = min(tb + tokens_per_cta, a.T);
+  if (tb >= te) return;
+  float4* g4 = reinterpret_cast<float4*>(a.g);
+  const float4* c4 = reinterpret_cast<const float4*>(coef);
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+
+  int64_t t = tb;
+  while (t < te) {
+    const int l = microbatch_of(a.off, a.M, t);
+    const int64_t lo = __ldg(a.off + l), hi = __ldg(a.off + l + 1);
+    // Malformed offsets (off[M] < T) must not stall the loop: tokens past
+    // the last boundary are treated as the last microbatch's.
+    const int64_t seg_end = (hi > t) ? min(te, hi) : te;
+
+    // ---- coefficients of microbatch l
+    __syncthreads();  // previous segment finished reading coef
+    const double n = (double)(hi - lo);
+    const double fbar = (double)a.K * n / (double)E;
+    double rho = 0.0;
+    if (threadIdx.x < E && n > 0.0)
+      rho = (double)__ldg(a.loads + (int64_t)l * E + threadIdx.x) / fbar - 1.0;
+    double amax = fabs(rho);
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) amax = fmax(amax, __shfl_xor_sync(kFull, amax, d));
+    if (lane == 0) red[wid] = amax;
+    __syncthreads();
+    double rmax = red[0];
+    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) rmax = fmax(rmax, red[w]);
+    double sigma = 1.0;
+    if (a.c > 0.0f) {
+      const double xi = rmax / (double)a.c;
+      sigma = (xi == 0.0) ? 1.0 : tanh(xi) / xi;
+    }
+    if (threadIdx.x < E) coef[threadIdx.x] = __double2float_rn((double)a.eta * sigma * rho);
+    __syncthreads();
+
+    // ---- stream grad_s[t .. seg_end) in float4 units
+    const int64_t i0 = t * E4, i1 = seg_end * E4;
+    const int S = blockDim.x;
+    const int dcol = S % E4;
+    int col = threadIdx.x % E4;
+    int64_t i = i0 + threadIdx.x;
+    for (; i + (int64_t)(kLeiUnroll - 1) * S < i1; i += (int64_t)kLeiUnroll * S) {
+      float4 v[kLeiUnroll];
+      int cc[kLeiUnroll];
+#pragma unroll
+      for (int u = 0; u < kLeiUnroll; ++u) {
+        v[u] = __ldcs(g4 + i + (int64_t)u * S);
+        cc[u] = col;
+        col += dcol;
+        if (col >= E4) col -= E4;
+      }
+#pragma unroll
+      for (int u = 0; u < kLeiUnroll; ++u) {
+        const float4 cf = c4[cc[u]];
+        v[u].x = __fadd_rn(v[u].x, cf.x);
+        v[u].y = __fadd_rn(v[u].y, cf.y);
+        v[u].z = __fadd_rn(v[u].z, cf.z);
+        v[u].w = __fadd_rn(v[u].w, cf.w);
+        __stcs(g4 + i + (int64_t)u * S, v[u]);
+      }
+    }
+    for (; i < i1; i += S) {
+      float4 v = __ldcs(g4 + i);
+      const float4 cf = c4[col];
+      v.x = __fadd_rn(v.x, cf.x);
+      v.y = __fadd_rn(v.y, cf.y);
+      v.z = __fadd_rn(v.z, cf.z);
+      v.w = __fadd_rn(v.w, cf.w);
+      __stcs(g4 + i, v);
+      col += dcol;
+      if (col >= E4) col -= E4;
+    }
+    t = seg_end;
+  }
+}
+
+}  // namespace
+
+int launch_lei(const LeiArgs& a, cudaStream_t s) {
+  DeviceInfo di;
+  if (int rc = device_info(&di)) return rc;
+  int64_t grid = (int64_t)di.sm_count * 8;
+  // at least 256 tokens per CTA so the per-microbatch prologue stays cheap
+  const int64_t max_grid = (a.T + 255) / 256;
+  if (grid > max_grid) grid = max_grid;
+  if (grid < 1) grid = 1;
+  const int64_t tpc = (a.T + grid - 1) / grid;
+  lei_kernel<<<(unsigned)grid, kLeiThreads, 0, s>>>(a, tpc);
+  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+}
+
+}  // namespace eqb

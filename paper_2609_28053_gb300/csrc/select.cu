@@ -1,0 +1,100 @@
+// select.cu -- Algorithm 1 steps 3, 5, 6 and the Eq. (2) centering
+// (arXiv 2609.28053, Sec. 2 and App. C).
+//
+// One warp per expert scans its 256 bins: each lane owns 8 consecutive
+// bins, a warp-wide inclusive prefix sum locates the lane whose range
+// reaches the rank, and that lane walks its 8 bins.
+//   pass 1: u_e = min{u : sum_{j<=u} H[e][j] >= r},  rho_e = r - sum_{j<u_e} H[e][j]
+//   pass 2: v_e = min{v : sum_{j<=v} L[e][j] >= rho_e},
+//           q_hat_e = kappa^{-1}((u_e << 8) | v_e)   (a zero returned as +0)
+// The bias update sums q_hat in fp64 in ascending expert order on one
+// thread, divides by E, and subtracts: the same operations in the same
+// order as the definition, so the result is reproducible bit for bit.
+#include "eqb_device.cuh"
+
+namespace eqb {
+
+namespace {
+
+__global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__ hist, int E, int pass,
+                                                     int64_t r, uint8_t* __restrict__ u,
+                                                     int32_t* __restrict__ rho,
+                                                     uint16_t* __restrict__ q_hat, int32_t* err) {
+  const int lane = threadIdx.x & 31;
+  const int e = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (e >= E) return;
+  const int32_t* h = hist + (int64_t)e * 256 + lane * 8;
+  int64_t cnt[8];
+  int64_t local = 0;
+#pragma unroll
+  for (int j = 0; j < 8; ++j) {
+    cnt[j] = h[j];
+    local += cnt[j];
+  }
+  int64_t incl = local;
+#pragma unroll
+  for (int d = 1; d < 32; d <<= 1) {
+    const int64_t o = __shfl_up_sync(kFull, incl, d);
+    if (lane >= d) incl += o;
+  }
+  const int64_t excl = incl - local;
+  const int64_t target = (pass == 1) ? r : (int64_t)rho[e];
+  const unsigned hit = __ballot_sync(kFull, excl < target && target <= incl);
+  if (pass == 1 && ((lane == 0 && cnt[0] != 0) || (lane == 31 && cnt[7] != 0)))
+    raise_flag(err, kErrNonfinite);
+  if (hit == 0u || target < 1) {
+    if (lane == 0) {
+      raise_flag(err, kErrRank);
+      if (pass == 1) { u[e] = 255; rho[e] = 0; }
+      else q_hat[e] = 0x7fc0;  // NaN marks an unreachable rank
+    }
+    return;
+  }
+  if (lane == __ffs(hit) - 1) {
+    int64_t below = excl;
+#pragma unroll
+    for (int j = 0; j < 8; ++j) {
+      if (below + cnt[j] >= target) {
+        const int bin = lane * 8 + j;
+        if (pass == 1) {
+          u[e] = static_cast<uint8_t>(bin);
+          rho[e] = static_cast<int32_t>(target - below);
+        } else {
+          uint32_t q = kappa16_inv((static_cast<uint32_t>(u[e]) << 8) | static_cast<uint32_t>(bin));
+          if (q == 0x8000u) q = 0u;
+          q_hat[e] = static_cast<uint16_t>(q);
+        }
+        break;
+      }
+      below += cnt[j];
+    }
+  }
+}
+
+__global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, float* __restrict__ b_next) {
+  __shared__ double mean;
+  if (threadIdx.x == 0) {
+    double sum = 0.0;
+    for (int e = 0; e < E; ++e) sum = __dadd_rn(sum, (double)bf16_bits_to_f32(q_hat[e]));
+    mean = __ddiv_rn(sum, (double)E);
+  }
+  __syncthreads();
+  for (int e = threadIdx.x; e < E; e += blockDim.x)
+    b_next[e] = __double2float_rn(__dsub_rn((double)bf16_bits_to_f32(q_hat[e]), mean));
+}
+
+}  // namespace
+
+int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, int32_t* rho,
+                  uint16_t* q_hat, int32_t* err, cudaStream_t s) {
+  const int wpb = 8;
+  select_kernel<<<(E + wpb - 1) / wpb, wpb * 32, 0, s>>>(hist, E, pass, r, u, rho, q_hat, err);
+  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+}
+
+int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t s) {
+  bias_update_kernel<<<1, 256, 0, s>>>(q_hat, E, b_next);
+  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+}
+
+}  // namespace eqb

@@ -1,0 +1,111 @@
+"""The C-ABI library builds, loads without a GPU, exports every entry point
+that include/eqb.h declares, and rejects invalid calls on the host before
+any CUDA call (so these run on a CPU-only machine)."""
+import ctypes
+import os
+import re
+import shutil
+
+import pytest
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "eqb.h")
+
+pytestmark = pytest.mark.skipif(shutil.which("nvcc") is None and not os.path.exists(
+    os.path.join(ROOT, "paper_2609_28053_gb300", "libeqb.so")), reason="no nvcc and no prebuilt library")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    from paper_2609_28053_gb300 import build, _lib
+    build.build()
+    return _lib.load()
+
+
+def declared_functions():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    names = re.findall(r"^\s*(?:const\s+)?[A-Za-z_][\w\s\*]*?\b((?:eqb|lei)_\w+)\s*\(", src, re.M)
+    return sorted(set(names))
+
+
+def test_header_declares_the_paper_entry_points():
+    names = declared_functions()
+    for n in ("eqb_route_topk", "eqb_margin_hist_pass1", "eqb_margin_hist_pass2",
+              "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad", "eqb_target_rank"):
+        assert n in names
+
+
+def test_every_declared_symbol_is_exported(lib):
+    for n in declared_functions():
+        assert hasattr(lib, n), f"{n} declared in eqb.h but not exported"
+
+
+def test_status_strings_and_version(lib):
+    for code, name in [(0, b"EQB_OK"), (1, b"EQB_ERR_INVALID_ARG"), (2, b"EQB_ERR_UNSUPPORTED"),
+                       (3, b"EQB_ERR_CUDA"), (4, b"EQB_ERR_NONFINITE"), (5, b"EQB_ERR_RANK")]:
+        assert lib.eqb_status_string(code) == name
+    assert lib.eqb_version() >= 100
+
+
+def test_target_rank(lib):
+    assert lib.eqb_target_rank(2097152, 256, 8) == 65536
+    assert lib.eqb_target_rank(10, 8, 3) == 4
+    assert lib.eqb_target_rank(-1, 8, 3) == -1
+    assert lib.eqb_target_rank(10, 0, 3) == -1
+
+
+# A fake, well-aligned address: invalid calls must return before using it.
+FAKE = ctypes.c_void_p(0x10000)
+MISALIGNED = ctypes.c_void_p(0x10002)
+NULL = None
+INVALID, UNSUPPORTED = 1, 2
+
+
+def route(lib, z=FAKE, b=FAKE, T=64, E=64, K=8, off=FAKE, M=1, idx=FAKE, tau=FAKE, loads=FAKE,
+          hist=FAKE, err=FAKE):
+    return lib.eqb_route_topk(z, b, T, E, K, off, M, idx, tau, loads, hist, err, NULL)
+
+
+@pytest.mark.parametrize("kw,code", [
+    (dict(K=0), INVALID), (dict(K=64), INVALID), (dict(T=-1), INVALID), (dict(E=1), INVALID),
+    (dict(E=12), UNSUPPORTED), (dict(E=264), UNSUPPORTED), (dict(E=64, K=32), UNSUPPORTED),
+    (dict(T=1 << 31), UNSUPPORTED), (dict(z=NULL), INVALID), (dict(b=NULL), INVALID),
+    (dict(tau=NULL), INVALID), (dict(off=NULL), INVALID), (dict(M=0), INVALID),
+    (dict(z=MISALIGNED), INVALID), (dict(tau=MISALIGNED), INVALID),
+])
+def test_route_rejects(lib, kw, code):
+    assert route(lib, **kw) == code
+
+
+def test_route_zero_tokens_is_a_noop(lib):
+    assert route(lib, T=0) == 0
+
+
+def test_hist_and_select_reject(lib):
+    assert lib.eqb_margin_hist_pass1(NULL, FAKE, 10, 64, FAKE, NULL, NULL) == INVALID
+    assert lib.eqb_margin_hist_pass1(FAKE, FAKE, 10, 60, FAKE, NULL, NULL) == UNSUPPORTED
+    assert lib.eqb_margin_hist_pass1(FAKE, FAKE, 0, 64, FAKE, NULL, NULL) == 0
+    assert lib.eqb_margin_hist_pass2(FAKE, FAKE, 10, 64, NULL, FAKE, NULL) == INVALID
+    assert lib.eqb_margin_hist_pass2(MISALIGNED, FAKE, 10, 64, FAKE, FAKE, NULL) == INVALID
+    assert lib.eqb_select_quantile(FAKE, 64, 3, 5, FAKE, FAKE, FAKE, NULL, NULL) == INVALID
+    assert lib.eqb_select_quantile(FAKE, 64, 1, 0, FAKE, FAKE, NULL, NULL, NULL) == INVALID
+    assert lib.eqb_select_quantile(FAKE, 64, 2, 5, FAKE, FAKE, NULL, NULL, NULL) == INVALID
+    assert lib.eqb_select_quantile(FAKE, 300, 1, 5, FAKE, FAKE, NULL, NULL, NULL) == UNSUPPORTED
+    assert lib.eqb_bias_update(FAKE, 0, FAKE, NULL) == INVALID
+    assert lib.eqb_bias_update(FAKE, 257, FAKE, NULL) == UNSUPPORTED
+
+
+def test_lei_rejects(lib):
+    f = lib.lei_inject_grad
+    assert f(NULL, FAKE, FAKE, 1, 10, 64, 8, ctypes.c_float(1.0), ctypes.c_float(1.0), NULL) == INVALID
+    assert f(FAKE, FAKE, FAKE, 0, 10, 64, 8, ctypes.c_float(1.0), ctypes.c_float(1.0), NULL) == INVALID
+    assert f(MISALIGNED, FAKE, FAKE, 1, 10, 64, 8, ctypes.c_float(1.0), ctypes.c_float(1.0), NULL) == INVALID
+    assert f(FAKE, FAKE, FAKE, 1, 10, 64, 8, ctypes.c_float(float("nan")), ctypes.c_float(1.0), NULL) == INVALID
+    assert f(FAKE, FAKE, FAKE, 1, 0, 64, 8, ctypes.c_float(1.0), ctypes.c_float(1.0), NULL) == 0
+
+
+def test_binding_fails_loudly_without_library(tmp_path):
+    from paper_2609_28053_gb300 import _lib
+    with pytest.raises(RuntimeError, match="no CPU fallback"):
+        _lib.load(str(tmp_path / "missing.so"))

@@ -1,0 +1,325 @@
+"""GPU parity: the CUDA path (through the C ABI) against the CPU oracle on the
+same seeded inputs.  Bit-exact for top-K indices, cutoffs, loads, both
+histograms, u, rho, the quantiles and the bias; LEI gradients within
+|d| <= 1e-7 + 1e-5 |g_ref|."""
+import numpy as np
+import pytest
+import torch
+
+import brute
+import oracle
+import paper_2609_28053_gb300 as eqb
+from eqb_workloads import (SHAPES, bits, even_offsets, make_bias, make_grad, make_logits,
+                           prior_batch_logits, ragged_offsets)
+from gpu_harness import Guarded, bits_f32, gpu_forward, oracle_forward, to_dev_bf16
+
+pytestmark = pytest.mark.gpu
+
+LEI_ATOL, LEI_RTOL = 1e-7, 1e-5
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib(cuda_ok):
+    eqb.load()
+
+
+def assert_forward_equal(g, o, check_hist=True):
+    assert np.array_equal(g["idx"], o["idx"]), "top-K indices differ"
+    assert np.array_equal(bits_f32(g["tau"]), bits_f32(o["tau"])), "tau differs"
+    assert np.array_equal(g["loads"], o["loads"]), "loads differ"
+    if check_hist:
+        assert np.array_equal(g["H"], o["H"]), "coarse histogram differs"
+        assert np.array_equal(g["u"], o["u"]) and np.array_equal(g["rho"], o["rho"])
+        assert np.array_equal(g["L"], o["L"]), "fine histogram differs"
+    assert np.array_equal(g["q"], o["q"]), "quantile differs"
+    assert np.array_equal(bits_f32(g["b_next"]), bits_f32(o["b_next"])), "bias update differs"
+    assert g["err"][0] == 0
+
+
+def rand_case(T, E, seed, scale=1.0, bias_scale=0.3, ties=False):
+    rng = np.random.default_rng(seed)
+    if ties:
+        v = rng.integers(-2, 3, size=(T, E)).astype(np.float32) * 0.25
+        b = np.zeros(E, np.float32)
+    else:
+        v = (rng.standard_normal((T, E)) * scale).astype(np.float32)
+        b = (rng.standard_normal(E) * bias_scale).astype(np.float32)
+    return brute.bf16_bits_from_f32(v), b
+
+
+# ------------------------------------------------------------- edge shapes
+
+@pytest.mark.parametrize("T", [1, 31, 32, 33, 1000, 4099])
+@pytest.mark.parametrize("E,K", [(8, 1), (8, 2), (8, 7), (16, 3), (24, 5), (64, 6), (64, 8),
+                                 (128, 8), (256, 6), (256, 8), (256, 15), (256, 31), (40, 31)])
+def test_forward_small_shapes(T, E, K):
+    z, b = rand_case(T, E, seed=T * 1000 + E * 10 + K)
+    off = ragged_offsets(T, 3, seed=T + E) if T > 3 else np.array([0, T], np.int64)
+    assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
+
+
+@pytest.mark.parametrize("E,K", [(8, 2), (64, 8), (256, 8), (256, 20)])
+def test_forward_exact_ties(E, K):
+    """Integer-valued logits with b = 0: most scores tie, so the candidate
+    lists overflow and the exact fallback decides by lower index."""
+    z, b = rand_case(517, E, seed=E + K, ties=True)
+    off = np.array([0, 200, 200, 517], np.int64)  # includes an empty microbatch
+    assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
+
+
+def test_forward_constant_rows():
+    T, E, K = 300, 64, 8
+    z = np.full((T, E), brute.bf16_bits_from_f32(np.float32([0.75]))[0], np.uint16)
+    z[::7] = brute.bf16_bits_from_f32(np.float32([-1.5]))[0]
+    b = np.zeros(E, np.float32)
+    off = np.array([0, T], np.int64)
+    assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
+
+
+def test_forward_signed_zero_subnormal_and_large_values():
+    rng = np.random.default_rng(5)
+    T, E, K = 777, 64, 8
+    v = (rng.standard_normal((T, E))).astype(np.float32)
+    v[rng.random((T, E)) < 0.1] = 0.0
+    v[rng.random((T, E)) < 0.1] = -0.0
+    v[rng.random((T, E)) < 0.05] = (rng.standard_normal(1) * 1e-39).astype(np.float32)[0]
+    v[rng.random((T, E)) < 0.02] = 1e30
+    v[rng.random((T, E)) < 0.02] = -1e30
+    z = brute.bf16_bits_from_f32(v)
+    b = (rng.standard_normal(E) * 1e-38).astype(np.float32)
+    b[::5] = -0.0
+    off = np.array([0, 400, T], np.int64)
+    assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
+
+
+# ------------------------------------------------------------- configs
+
+def config_inputs(name, T=None):
+    sh = SHAPES[name]
+    T = sh.T if T is None else T
+    z = bits(make_logits(name, T=T))
+    if name == "mid":
+        zp = bits(prior_batch_logits(name, T=T))
+        b = oracle.eqb_step(zp, np.zeros(sh.E, np.float32), sh.K)["b_next"]
+    else:
+        b = make_bias(name).numpy()
+    return z, b, even_offsets(T, sh.M), sh.K
+
+
+@pytest.mark.parametrize("name", ["tiny", "tie", "mid"])
+def test_config_forward(name):
+    z, b, off, K = config_inputs(name)
+    assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
+
+
+def test_tie_config_repartitioned():
+    """Tie-heavy config: the quantile is the same for P = 8, 1, 3, 13 and 64
+    uneven partitions and for a token permutation: histograms of
+    per-partition calls accumulate into the same device buffers."""
+    z, b, off, K = config_inputs("tie")
+    T, E = z.shape
+    ref = oracle_forward(z, b, K, off)
+    r = ref["r"]
+    rng = np.random.default_rng(0)
+    for P, perm in [(8, False), (1, False), (3, False), (13, True), (64, True)]:
+        order = rng.permutation(T) if perm else np.arange(T)
+        zz = z[order]
+        cuts = np.sort(rng.choice(np.arange(1, T), size=P - 1, replace=False)) if P > 1 else []
+        bounds = np.concatenate([[0], cuts, [T]]).astype(np.int64)
+        zd = to_dev_bf16(zz)
+        bt = torch.from_numpy(b).cuda()
+        tau = torch.empty(T, dtype=torch.float32, device="cuda")
+        H = torch.zeros((E, 256), dtype=torch.int32, device="cuda")
+        L = torch.zeros_like(H)
+        u = torch.zeros(E, dtype=torch.uint8, device="cuda")
+        rho = torch.zeros(E, dtype=torch.int32, device="cuda")
+        q = torch.zeros(E, dtype=torch.bfloat16, device="cuda")
+        err = torch.zeros(1, dtype=torch.int32, device="cuda")
+        for p in range(P):
+            a, c = int(bounds[p]), int(bounds[p + 1])
+            eqb.eqb_route_topk(zd[a:c], bt, K, None, None, tau[a:c], None, H, err)
+        eqb.eqb_select_quantile(H, 1, r, u, rho, None, err)
+        for p in range(P):
+            a, c = int(bounds[p]), int(bounds[p + 1])
+            eqb.eqb_margin_hist_pass2(zd[a:c], tau[a:c], u, L)
+        eqb.eqb_select_quantile(L, 2, r, u, rho, q, err)
+        torch.cuda.synchronize()
+        assert np.array_equal(H.cpu().numpy(), ref["H"])
+        assert np.array_equal(q.view(torch.int16).cpu().numpy().view(np.uint16), ref["q"])
+        assert err.item() == 0
+
+
+@pytest.mark.slow
+def test_global_config_full_size_sampled():
+    """Full size (T = 2,097,152, E = 256, K = 8, M = 64): every token's top-K
+    and cutoff, all loads, and the exact quantile of 16 sampled experts
+    against the oracle; the launch configuration is the benchmark's."""
+    name = "global"
+    sh = SHAPES[name]
+    zt = make_logits(name, device="cuda")
+    z = bits(zt)
+    b = make_bias(name, device="cuda").cpu().numpy()
+    off = even_offsets(sh.T, sh.M)
+    g = gpu_forward(z, b, sh.K, off)
+    experts = np.random.default_rng(1).choice(sh.E, 16, replace=False)
+    o = oracle_forward(z, b, sh.K, off, experts=experts)
+    assert np.array_equal(g["idx"], o["idx"])
+    assert np.array_equal(bits_f32(g["tau"]), bits_f32(o["tau"]))
+    assert np.array_equal(g["loads"], o["loads"])
+    assert np.array_equal(g["q"][experts], o["q"])
+    # histogram totals: every expert saw all T margins
+    assert np.all(g["H"].sum(1) == sh.T)
+    assert np.all(g["L"].sum(1) >= g["rho"])
+    assert g["err"][0] == 0
+
+
+@pytest.mark.slow
+def test_router_config_three_steps_on_torch_logits():
+    """Router config: z = bf16(x W_r^T) (here from torch's matmul), bias
+    iterated for 3 steps from b^(0) = 0 with fresh activations; each step's
+    GPU bias feeds the next GPU step and the oracle's feeds the oracle's, so
+    bit-exact agreement at every step pins the whole chain.  Reduced T."""
+    from eqb_workloads import make_router_inputs
+    sh = SHAPES["router"]
+    T = 65536
+    b_gpu = np.zeros(sh.E, np.float32)
+    b_or = np.zeros(sh.E, np.float32)
+    off = even_offsets(T, sh.M)
+    for step in range(3):
+        x, W = make_router_inputs(T=T, step=step, device="cuda")
+        z = bits((x.float() @ W.float().t()).to(torch.bfloat16))
+        g = gpu_forward(z, b_gpu, sh.K, off)
+        o = oracle_forward(z, b_or, sh.K, off)
+        assert_forward_equal(g, o)
+        b_gpu, b_or = g["b_next"], o["b_next"]
+
+
+# ------------------------------------------------------------- per-call units
+
+def test_standalone_pass1_matches_oracle_counts():
+    z, b = rand_case(3000, 128, seed=11)
+    _, tau, _ = oracle.route(z, b, 8)
+    H_ref = oracle.hist_hi(z, tau)
+    H = Guarded((128, 256), torch.int32)
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    eqb.eqb_margin_hist_pass1(to_dev_bf16(z), torch.from_numpy(tau).cuda(), H.view, err)
+    torch.cuda.synchronize()
+    assert H.intact() and np.array_equal(H.view.cpu().numpy(), H_ref) and err.item() == 0
+
+
+def test_select_and_bias_from_oracle_histograms():
+    z, b = rand_case(5000, 64, seed=12)
+    K = 6
+    _, tau, _ = oracle.route(z, b, K)
+    r = oracle.target_rank(5000, 64, K)
+    H = oracle.hist_hi(z, tau)
+    u, rho = oracle.select_hi(H, r)
+    L = oracle.hist_lo(z, tau, u)
+    q = oracle.select_lo(L, u, rho)
+    bn = oracle.bias_update(q)
+    ud = torch.zeros(64, dtype=torch.uint8, device="cuda")
+    rd = torch.zeros(64, dtype=torch.int32, device="cuda")
+    qd = torch.zeros(64, dtype=torch.bfloat16, device="cuda")
+    bd = torch.zeros(64, dtype=torch.float32, device="cuda")
+    eqb.eqb_select_quantile(torch.from_numpy(H).cuda(), 1, r, ud, rd)
+    torch.cuda.synchronize()
+    assert np.array_equal(ud.cpu().numpy(), u) and np.array_equal(rd.cpu().numpy(), rho)
+    eqb.eqb_select_quantile(torch.from_numpy(L).cuda(), 2, r, torch.from_numpy(u).cuda(),
+                            torch.from_numpy(rho).cuda(), qd)
+    eqb.eqb_bias_update(torch.from_numpy(q.view(np.int16)).view(torch.bfloat16).cuda(), bd)
+    torch.cuda.synchronize()
+    assert np.array_equal(qd.view(torch.int16).cpu().numpy().view(np.uint16), q)
+    assert np.array_equal(bits_f32(bd.cpu().numpy()), bits_f32(bn))
+
+
+@pytest.mark.parametrize("T,E,K,M", [(4096, 8, 2, 4), (1001, 64, 8, 5), (65536, 64, 8, 8),
+                                     (33, 256, 8, 2), (5000, 24, 3, 7)])
+@pytest.mark.parametrize("eta,c", [(1.0, 0.5), (0.25, 4.0), (0.02, 0.0), (2e-5, 1.0)])
+def test_lei_matches_oracle(T, E, K, M, eta, c):
+    z, b = rand_case(T, E, seed=T + E)
+    off = ragged_offsets(T, M, seed=E)
+    _, _, loads = oracle.route(z, b, K, off)
+    g = (np.random.default_rng(T).standard_normal((T, E)) * 0.1).astype(np.float32)
+    g_ref, _ = oracle.lei(g, loads, off, K, eta, c)
+    G = Guarded((T, E), torch.float32)
+    G.view.copy_(torch.from_numpy(g))
+    eqb.lei_inject_grad(G.view, torch.from_numpy(loads).cuda(), torch.from_numpy(off).cuda(), K, eta, c)
+    torch.cuda.synchronize()
+    assert G.intact()
+    got = G.view.cpu().numpy()
+    assert np.all(np.abs(got.astype(np.float64) - g_ref) <= LEI_ATOL + LEI_RTOL * np.abs(g_ref))
+
+
+def test_lei_eta_zero_and_balanced_are_identity():
+    T, E, K = 2048, 64, 8
+    g = (np.random.default_rng(1).standard_normal((T, E)) * 0.1).astype(np.float32)
+    off = np.array([0, 1024, 2048], np.int64)
+    loads = np.full((2, E), K * 1024 // E, np.int32)  # perfectly balanced
+    for eta, ld in [(0.0, np.random.default_rng(2).integers(0, 300, (2, E)).astype(np.int32)),
+                    (1.0, loads)]:
+        G = torch.from_numpy(g).cuda()
+        eqb.lei_inject_grad(G, torch.from_numpy(ld).cuda(), torch.from_numpy(off).cuda(), K, eta, 1.0)
+        torch.cuda.synchronize()
+        assert np.array_equal(G.cpu().numpy(), g)
+
+
+def test_lei_global_config_full_size_sampled():
+    name = "global"
+    sh = SHAPES[name]
+    T, E = sh.T, sh.E
+    off = even_offsets(T, sh.M)
+    rng = np.random.default_rng(3)
+    loads = rng.multinomial(sh.K * (T // sh.M), np.ones(E) / E, size=sh.M).astype(np.int32)
+    G = make_grad(name, device="cuda")
+    g0 = G.clone()
+    eqb.lei_inject_grad(G, torch.from_numpy(loads).cuda(), torch.from_numpy(off).cuda(), sh.K, 2e-5, 1.0)
+    rows = np.sort(rng.choice(T, 4096, replace=False))
+    got = G[torch.from_numpy(rows).cuda()].cpu().numpy()
+    g_rows = g0[torch.from_numpy(rows).cuda()].cpu().numpy()
+    _, a = oracle.lei(None, loads, off, sh.K, 2e-5, 1.0)
+    mb = np.searchsorted(off, rows, side="right") - 1
+    want = (g_rows.astype(np.float64) + a[mb]).astype(np.float32)
+    assert np.all(np.abs(got.astype(np.float64) - want) <= LEI_ATOL + LEI_RTOL * np.abs(want))
+
+
+# ------------------------------------------------------------- device-side errors
+
+def test_nonfinite_logit_sets_flag():
+    z, b = rand_case(500, 64, seed=3)
+    z[123, 7] = 0x7fc0  # NaN
+    g = gpu_forward(z, b, 8, np.array([0, 500], np.int64))
+    assert g["err"][0] == 4
+
+
+def test_infinite_logit_sets_flag():
+    z, b = rand_case(500, 64, seed=4)
+    z[10, 3] = 0xff80  # -inf
+    g = gpu_forward(z, b, 8, np.array([0, 500], np.int64))
+    assert g["err"][0] == 4
+
+
+def test_nonfinite_bias_sets_flag():
+    z, b = rand_case(100, 64, seed=5)
+    b[9] = np.inf
+    g = gpu_forward(z, b, 8, np.array([0, 100], np.int64))
+    assert g["err"][0] == 4
+
+
+def test_huge_margin_sets_flag():
+    z, b = rand_case(100, 64, seed=6)
+    z[5, :] = brute.bf16_bits_from_f32(np.float32([3e38]))[0]
+    z[5, 0] = brute.bf16_bits_from_f32(np.float32([-3e38]))[0]
+    g = gpu_forward(z, b, 8, np.array([0, 100], np.int64))
+    assert g["err"][0] == 4
+
+
+def test_unreachable_rank_sets_flag():
+    z, b = rand_case(100, 64, seed=7)
+    _, tau, _ = oracle.route(z, b, 8)
+    H = oracle.hist_hi(z, tau)
+    u = torch.zeros(64, dtype=torch.uint8, device="cuda")
+    rho = torch.zeros(64, dtype=torch.int32, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    eqb.eqb_select_quantile(torch.from_numpy(H).cuda(), 1, 101, u, rho, None, err)
+    torch.cuda.synchronize()
+    assert err.item() == 5
