@@ -16,8 +16,8 @@
 //   B. candidates: every e with s_e >= theta (a superset of the top-(K+1)
 //      set, ties included) is appended, in ascending e, to a per-lane list.
 //   C. exact selection: stable insertion of the candidates into a sorted
-//      (K+1)-list, strictly-greater comparisons, so equal scores keep the
-//      lower expert index first.  A lane whose list overflows (many ties
+//      (K+1)-list (a new candidate goes after equal scores, displaced
+//      entries shift down), so equal scores keep the lower index first.  A lane whose list overflows (many ties
 //      at theta) falls back to K+1 exact scans of its row.
 // Loads are counted in per-warp shared counters for the warp's current
 // microbatch and flushed to global memory when the microbatch changes; each
@@ -61,11 +61,16 @@ __device__ __forceinline__ void sort_desc(float (&a)[N]) {
   }
 }
 
+// Insert (s, e) into the descending list (v, id).  Candidates arrive in
+// ascending e, so a new element goes after equal scores (strict compare);
+// once it has been placed, every later slot shifts down unconditionally.
 template <int KP1>
 __device__ __forceinline__ void insert_sorted(float (&v)[KP1], int (&id)[KP1], float s, int e) {
+  bool moved = false;
 #pragma unroll
   for (int j = 0; j < KP1; ++j) {
-    const bool gt = s > v[j];
+    const bool gt = moved || s > v[j];
+    moved = gt;
     const float tv = v[j];
     const int ti = id[j];
     v[j] = gt ? s : tv;

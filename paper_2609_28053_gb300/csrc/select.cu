@@ -7,9 +7,8 @@
 //   pass 1: u_e = min{u : sum_{j<=u} H[e][j] >= r},  rho_e = r - sum_{j<u_e} H[e][j]
 //   pass 2: v_e = min{v : sum_{j<=v} L[e][j] >= rho_e},
 //           q_hat_e = kappa^{-1}((u_e << 8) | v_e)   (a zero returned as +0)
-// The bias update sums q_hat in fp64 in ascending expert order on one
-// thread, divides by E, and subtracts: the same operations in the same
-// order as the definition, so the result is reproducible bit for bit.
+// The bias update reproduces the definition's fp64 sum in ascending expert
+// order bit for bit (see bias_update_kernel), divides by E and subtracts.
 #include "eqb_device.cuh"
 
 namespace eqb {
@@ -71,12 +70,52 @@ __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__
   }
 }
 
+// Exponent range of a non-zero bf16 pattern: [ulp exponent, leading-bit exponent].
+__device__ __forceinline__ void bf16_exp_range(uint32_t x, int& lo, int& hi) {
+  const int ex = (x >> 7) & 0xff;
+  const uint32_t man = x & 0x7f;
+  if (ex != 0) { lo = ex - 127 - 7; hi = ex - 127; }
+  else { lo = -133; hi = -134 + (32 - __clz(man)); }  // subnormal
+}
+
+// b_next = q_hat - mean(q_hat), mean = (sum in ascending e, fp64) / E.
+// If every non-zero q_hat lies within a window where all partial sums of up
+// to 256 terms are exact in fp64 (leading-bit exponent - ulp exponent + 9 <=
+// 52), any summation order gives the exact sum, so a warp tree reduction
+// reproduces the sequential sum bit for bit.  Otherwise one thread sums in
+// ascending order.
 __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, float* __restrict__ b_next) {
   __shared__ double mean;
-  if (threadIdx.x == 0) {
-    double sum = 0.0;
-    for (int e = 0; e < E; ++e) sum = __dadd_rn(sum, (double)bf16_bits_to_f32(q_hat[e]));
-    mean = __ddiv_rn(sum, (double)E);
+  if (threadIdx.x < 32) {
+    const int lane = threadIdx.x;
+    double part = 0.0;
+    int lo = 1 << 20, hi = -(1 << 20);
+    for (int e = lane; e < E; e += 32) {
+      const uint32_t x = q_hat[e];
+      if ((x & 0x7fffu) != 0u) {
+        int l, h;
+        bf16_exp_range(x, l, h);
+        lo = min(lo, l);
+        hi = max(hi, h);
+      }
+      part = __dadd_rn(part, (double)bf16_bits_to_f32(x));
+    }
+#pragma unroll
+    for (int d = 16; d > 0; d >>= 1) {
+      lo = min(lo, __shfl_xor_sync(kFull, lo, d));
+      hi = max(hi, __shfl_xor_sync(kFull, hi, d));
+    }
+    double sum;
+    if (hi - lo + 9 <= 52 || hi < lo) {
+#pragma unroll
+      for (int d = 16; d > 0; d >>= 1) part = __dadd_rn(part, __shfl_xor_sync(kFull, part, d));
+      sum = part;
+    } else {
+      sum = 0.0;
+      if (lane == 0)
+        for (int e = 0; e < E; ++e) sum = __dadd_rn(sum, (double)bf16_bits_to_f32(q_hat[e]));
+    }
+    if (lane == 0) mean = __ddiv_rn(sum, (double)E);
   }
   __syncthreads();
   for (int e = threadIdx.x; e < E; e += blockDim.x)

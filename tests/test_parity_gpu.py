@@ -323,3 +323,26 @@ def test_unreachable_rank_sets_flag():
     eqb.eqb_select_quantile(torch.from_numpy(H).cuda(), 1, 101, u, rho, None, err)
     torch.cuda.synchronize()
     assert err.item() == 5
+
+
+@pytest.mark.parametrize("kind", ["narrow", "wide", "subnormal", "zeros"])
+def test_bias_update_exact_against_oracle(kind):
+    """The fixed-order fp64 centering of Eq. (2) reproduces the oracle bit for
+    bit both when a tree sum is provably exact (narrow exponent span) and
+    when it is not (wide span forces the ascending sequential sum)."""
+    rng = np.random.default_rng(hash(kind) % 1000)
+    E = 256
+    v = (rng.standard_normal(E) * 3).astype(np.float32)
+    if kind == "wide":
+        v[::17] *= np.float32(1e30)
+        v[5::23] *= np.float32(1e-30)
+    elif kind == "subnormal":
+        v[::3] = np.float32(1e-39)
+    elif kind == "zeros":
+        v[:] = 0.0
+    q = brute.bf16_bits_from_f32(v)
+    want = oracle.bias_update(q)
+    bd = torch.zeros(E, dtype=torch.float32, device="cuda")
+    eqb.eqb_bias_update(torch.from_numpy(q.view(np.int16)).view(torch.bfloat16).cuda(), bd)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits_f32(bd.cpu().numpy()), bits_f32(want))
