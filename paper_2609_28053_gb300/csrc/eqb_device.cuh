@@ -78,3 +78,62 @@ __device__ __forceinline__ void raise_flag(int32_t* err, int code) {
 }
 
 }  // namespace eqb
+
+namespace eqb {
+
+// ---- packed bf16x2 helpers (two bf16 values per 32-bit word)
+
+__device__ __forceinline__ uint32_t hadd2_bf16(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("add.rn.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+__device__ __forceinline__ uint32_t hmax2_nan_bf16(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.NaN.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// Per half: 0xffff where a >= b, else 0 (NaN compares false).
+__device__ __forceinline__ uint32_t hge2_bf16(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("set.ge.u32.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
+// Byte permute with the PTX default mode (a selector nibble with bit 3 set
+// replicates the sign bit of the selected byte).
+__device__ __forceinline__ uint32_t prmt(uint32_t a, uint32_t b, uint32_t sel) {
+  uint32_t r;
+  asm("prmt.b32 %0, %1, %2, %3;" : "=r"(r) : "r"(a), "r"(b), "r"(sel));
+  return r;
+}
+
+// Internal keys of two packed bf16 patterns: kappa(x) ^ 0x8000 per half,
+// i.e. x ^ 0x7fff for negative x, x otherwise.  The internal high byte is the
+// true high byte ^ 0x80; the low byte is the true low byte.
+__device__ __forceinline__ uint32_t kappa2_internal(uint32_t m) {
+  const uint32_t sm = prmt(m, 0u, 0xBB99u);  // 0xffff per negative half
+  return m ^ (sm & 0x7fff7fffu);
+}
+
+// bf16 pattern of fp32 x rounded toward -inf / +inf (exact values kept).
+__device__ __forceinline__ uint32_t bf16_round_down(float x) {
+  const uint32_t u = __float_as_uint(x);
+  const uint32_t hi = u >> 16;
+  if ((u & 0xffffu) == 0u) return hi;
+  return (u & 0x80000000u) ? hi + 1u : hi;
+}
+__device__ __forceinline__ uint32_t bf16_round_up(float x) {
+  const uint32_t u = __float_as_uint(x);
+  const uint32_t hi = u >> 16;
+  if ((u & 0xffffu) == 0u) return hi;
+  return (u & 0x80000000u) ? hi : hi + 1u;
+}
+
+__device__ __forceinline__ void red_shared_add(uint32_t saddr, uint32_t v) {
+  asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(saddr), "r"(v));
+}
+
+}  // namespace eqb

@@ -2,117 +2,145 @@
 // Sec. 3 and App. C, steps 1 and 4).
 //
 // Both passes recompute every routing margin m = bf16_rne(tau_t - fp32(z))
-// from z and tau instead of reading a stored margin array (Sec. 3: "the
-// second pass simply rescans local margins").  The order-preserving key is
-// k = kappa(m) (negative patterns complemented, others get the sign bit);
-// pass 1 counts the high byte k >> 8, pass 2 counts the low byte k & 0xff of
-// the margins whose high byte equals the selected u_e.
+// from z and tau instead of reading a stored margin array (Sec. 3: the second
+// pass rescans the local margins).  Keys are kappa(m) (negative patterns
+// complemented, others with the sign bit set).  Pass 1 counts the high byte of
+// every key; pass 2 counts the low byte of the keys whose high byte is u_e.
 //
-// Layout: the grid is (expert tiles) x (token ranges).  A CTA owns ET
-// experts (ET = 64 when E allows) and keeps their ET x 256 int32 bins in
-// shared memory (64 KiB), so three CTAs fit per SM.  Within a warp, ET/8
-// lanes cover one token's ET experts with one 16-byte load each, so each
-// load instruction of the warp reads whole contiguous row segments.  The
-// bins of expert e_l are stored XOR-swizzled by (e_l >> 3): the lanes of one
-// token hit distinct banks even when their margins share a bin.  At the end
-// every CTA adds its non-zero bins into the global [E,256] histogram, which
-// is how token partitions are summed in device memory.
+// Work per element is kept to a handful of instructions by working on packed
+// pairs: one 32-bit word of z holds two experts, their two margins are
+// rounded with one cvt.rn.bf16x2, and one PRMT (sign replicate) plus one LOP3
+// give both internal keys (kappa ^ 0x8000, so the stored high byte is the
+// true one ^ 0x80 and is translated back at the flush).
+//
+// Bins: a CTA owns ET experts (all E when E <= 256 is a power of two) and
+// keeps their 256 bins as 16-bit counters, two experts per 32-bit word: the
+// experts of one z word share a word, the even one in the low half, so the
+// increment is a constant.  ET * 512 bytes: 128 KiB for E = 256.  The ET/8
+// lanes covering one token each own 8 experts; lane c's rows start c words
+// past a 1 KiB boundary so equal bins of the 32 lanes fall in 32 banks.  A
+// counter gains at most one per token, so the CTA flushes (adds its non-zero
+// counters into the global int32 [E,256] histogram) at least every 65,535
+// tokens; the flush is also how token partitions are summed in device memory.
 #include "eqb_device.cuh"
 
 namespace eqb {
 
 namespace {
 
-constexpr int kHistThreads = 512;
 constexpr int kUnroll = 4;
+constexpr int64_t kFlushTokens = 65535;
+
+template <int LPT>
+struct HistLayout {
+  static constexpr int ET = LPT * 8;            // experts per CTA
+  static constexpr int TPS = 32 / LPT;          // tokens per warp step
+  static constexpr int kRows = ET / 2;          // one row per expert pair
+  static constexpr int kWords = kRows * 256 + LPT;
+  __host__ __device__ static int row_word(int row) { return row * 256 + (row >> 2); }
+};
 
 template <int PASS, int LPT>
-__global__ void __launch_bounds__(kHistThreads) hist_kernel(HistArgs a, int64_t tokens_per_cta) {
+__global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_per_cta) {
+  using Lay = HistLayout<LPT>;
   extern __shared__ __align__(16) uint32_t bins[];
-  constexpr int ET = LPT * 8;     // experts per CTA
-  constexpr int TPS = 32 / LPT;   // tokens per warp step
   const int E = a.E;
-  const int e0 = blockIdx.x * ET;
+  const int e0 = blockIdx.x * Lay::ET;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
   const int nw = blockDim.x >> 5;
-  const int c = lane % LPT;        // chunk of 8 experts inside the tile
-  const int tok = lane / LPT;      // token slot inside the warp step
+  const int c = lane % LPT;     // 8-expert chunk of the tile owned by this lane
+  const int tok = lane / LPT;   // token slot inside the warp step
 
-  for (int i = threadIdx.x; i < ET * 256; i += blockDim.x) bins[i] = 0;
-  uint32_t uu[8];
+  for (int i = threadIdx.x; i < Lay::kWords; i += blockDim.x) bins[i] = 0u;
+  // Shared address of this lane's first pair row; pair p adds p * 1 KiB.
+  const uint32_t base = static_cast<uint32_t>(__cvta_generic_to_shared(bins)) +
+                        4u * static_cast<uint32_t>(Lay::row_word(4 * c));
+  uint32_t sel[4] = {0, 0, 0, 0};
   if (PASS == 2) {
+    // internal high bytes (u ^ 0x80) of the selected bins, placed where the
+    // internal keys carry them: bits 8-15 (even expert) and 24-31 (odd).
 #pragma unroll
-    for (int j = 0; j < 8; ++j) uu[j] = a.u[e0 + c * 8 + j];
+    for (int p = 0; p < 4; ++p) {
+      const uint32_t ue = a.u[e0 + c * 8 + 2 * p] ^ 0x80u;
+      const uint32_t uo = a.u[e0 + c * 8 + 2 * p + 1] ^ 0x80u;
+      sel[p] = (ue << 8) | (uo << 24);
+    }
   }
   __syncthreads();
 
   const int64_t tb = (int64_t)blockIdx.y * tokens_per_cta;
   const int64_t te = min(tb + tokens_per_cta, a.T);
-  uint32_t* my = bins + (c * 8) * 256;  // row of expert c*8 + 0
-  const uint32_t sw = static_cast<uint32_t>(c);
-
-  for (int64_t base = tb + (int64_t)wid * TPS; base < te; base += (int64_t)nw * TPS * kUnroll) {
-    uint4 w[kUnroll];
-    float tt[kUnroll];
+  for (int64_t cb = tb; cb < te; cb += kFlushTokens) {
+    const int64_t ce = min(cb + kFlushTokens, te);
+    for (int64_t base_t = cb + (int64_t)wid * Lay::TPS; base_t < ce;
+         base_t += (int64_t)nw * Lay::TPS * kUnroll) {
+      uint4 w[kUnroll];
+      float tt[kUnroll];
 #pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t t = base + (int64_t)u * nw * TPS + tok;
-      if (t < te) {
-        w[u] = __ldcs(reinterpret_cast<const uint4*>(a.z + t * E + e0 + c * 8));
-        tt[u] = __ldg(a.tau + t);
-      } else {
-        w[u] = make_uint4(0, 0, 0, 0);
-        tt[u] = 0.f;
-      }
-    }
-#pragma unroll
-    for (int u = 0; u < kUnroll; ++u) {
-      const int64_t t = base + (int64_t)u * nw * TPS + tok;
-      if (t >= te) continue;
-      const float tv = tt[u];
-      uint32_t m[4];
-      m[0] = pack_bf16x2_rn(tv - bf16_lo(w[u].x), tv - bf16_hi(w[u].x));
-      m[1] = pack_bf16x2_rn(tv - bf16_lo(w[u].y), tv - bf16_hi(w[u].y));
-      m[2] = pack_bf16x2_rn(tv - bf16_lo(w[u].z), tv - bf16_hi(w[u].z));
-      m[3] = pack_bf16x2_rn(tv - bf16_lo(w[u].w), tv - bf16_hi(w[u].w));
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        const uint32_t x16 = (j & 1) ? (m[j >> 1] >> 16) : (m[j >> 1] & 0xffffu);
-        const uint32_t k = kappa16(x16);
-        if (PASS == 1) {
-          atomicAdd(my + j * 256 + ((k >> 8) ^ sw), 1u);
+      for (int u = 0; u < kUnroll; ++u) {
+        const int64_t t = base_t + (int64_t)u * nw * Lay::TPS + tok;
+        if (t < ce) {
+          w[u] = __ldcs(reinterpret_cast<const uint4*>(a.z + t * E + e0 + c * 8));
+          tt[u] = __ldg(a.tau + t);
         } else {
-          if ((k >> 8) == uu[j]) atomicAdd(my + j * 256 + ((k & 0xffu) ^ sw), 1u);
+          w[u] = make_uint4(0, 0, 0, 0);
+          tt[u] = 0.f;
+        }
+      }
+#pragma unroll
+      for (int u = 0; u < kUnroll; ++u) {
+        const int64_t t = base_t + (int64_t)u * nw * Lay::TPS + tok;
+        if (t >= ce) continue;
+        const float tv = tt[u];
+        const uint32_t zw[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+#pragma unroll
+        for (int p = 0; p < 4; ++p) {
+          const uint32_t m = pack_bf16x2_rn(tv - bf16_lo(zw[p]), tv - bf16_hi(zw[p]));
+          const uint32_t k = kappa2_internal(m);
+          const uint32_t row = base + 1024u * p;
+          if (PASS == 1) {
+            red_shared_add(row + 4u * prmt(k, 0u, 0x4441u), 1u);        // even expert
+            red_shared_add(row + 4u * (k >> 24), 0x10000u);              // odd expert
+          } else {
+            const uint32_t d = (k ^ sel[p]) & 0xff00ff00u;
+            if ((d & 0x0000ff00u) == 0u) red_shared_add(row + 4u * (k & 0xffu), 1u);
+            if ((d & 0xff000000u) == 0u) red_shared_add(row + 4u * prmt(k, 0u, 0x4442u), 0x10000u);
+          }
         }
       }
     }
-  }
-  __syncthreads();
-
-  for (int i = threadIdx.x; i < ET * 256; i += blockDim.x) {
-    const uint32_t v = bins[i];
-    if (v) {
-      const int el = i >> 8;
-      const int bin = (i & 255) ^ (el >> 3);
-      atomicAdd(a.hist + (int64_t)(e0 + el) * 256 + bin, static_cast<int>(v));
-      if (PASS == 1 && (bin == 0 || bin == 255)) raise_flag(a.err, kErrNonfinite);
+    __syncthreads();
+    // Flush: add every non-zero 16-bit counter to the global histogram.
+    for (int i = threadIdx.x; i < Lay::kRows * 256; i += blockDim.x) {
+      const int row = i >> 8, slot = i & 255;
+      const int wi = Lay::row_word(row) + slot;
+      const uint32_t v = bins[wi];
+      if (v) {
+        bins[wi] = 0u;
+        const int bin = (PASS == 1) ? (slot ^ 0x80) : slot;
+        const int ee = e0 + 2 * row;
+        if (v & 0xffffu) atomicAdd(a.hist + (int64_t)ee * 256 + bin, static_cast<int>(v & 0xffffu));
+        if (v >> 16) atomicAdd(a.hist + (int64_t)(ee + 1) * 256 + bin, static_cast<int>(v >> 16));
+        if (PASS == 1 && (bin == 0 || bin == 255)) raise_flag(a.err, kErrNonfinite);
+      }
     }
+    __syncthreads();
   }
 }
 
 template <int PASS, int LPT>
 int launch_hist_t(const HistArgs& a, cudaStream_t s) {
-  constexpr int ET = LPT * 8;
+  using Lay = HistLayout<LPT>;
   DeviceInfo di;
   if (int rc = device_info(&di)) return rc;
-  const int smem = ET * 256 * 4;
-  const int nE = a.E / ET;
+  const int smem = Lay::kWords * 4;
+  const int nE = a.E / Lay::ET;
   int ctas_per_sm = (228 * 1024 - 1024) / (smem + 1024);
-  if (ctas_per_sm > 4) ctas_per_sm = 4;
   if (ctas_per_sm < 1) ctas_per_sm = 1;
+  const int threads = ctas_per_sm == 1 ? 1024 : 512;
+  if (ctas_per_sm > 2048 / threads) ctas_per_sm = 2048 / threads;
   int64_t nT = ((int64_t)di.sm_count * ctas_per_sm + nE - 1) / nE;
-  // keep at least ~2048 tokens per CTA so the flush stays small
-  const int64_t max_nT = (a.T + 2047) / 2048;
+  const int64_t max_nT = (a.T + 2047) / 2048;  // keep >= ~2K tokens per CTA
   if (nT > max_nT) nT = max_nT;
   if (nT < 1) nT = 1;
   const int64_t tpc = (a.T + nT - 1) / nT;
@@ -120,12 +148,14 @@ int launch_hist_t(const HistArgs& a, cudaStream_t s) {
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
     return kErrCuda;
   dim3 grid((unsigned)nE, (unsigned)nT);
-  kern<<<grid, kHistThreads, smem, s>>>(a, tpc);
+  kern<<<grid, threads, smem, s>>>(a, tpc);
   return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
 }
 
 template <int PASS>
 int launch_hist_pass(const HistArgs& a, cudaStream_t s) {
+  if (a.E % 256 == 0) return launch_hist_t<PASS, 32>(a, s);
+  if (a.E % 128 == 0) return launch_hist_t<PASS, 16>(a, s);
   if (a.E % 64 == 0) return launch_hist_t<PASS, 8>(a, s);
   if (a.E % 32 == 0) return launch_hist_t<PASS, 4>(a, s);
   if (a.E % 16 == 0) return launch_hist_t<PASS, 2>(a, s);

@@ -2,44 +2,49 @@
 // (Sec. 2, Eq. 1 and the QB paragraph of arXiv 2609.28053).
 //
 // One thread owns one token.  A warp stages a tile of 32 consecutive token
-// rows of z (32 * E bf16, one contiguous block of global memory) in shared
-// memory with coalesced 16-byte cp.async copies, double-buffered so the next
-// tile streams in while the current one is processed.  Rows are padded to a
-// stride of 4 (mod 8) words, so the 32 lanes reading the same 16-byte column
-// chunk of their own rows hit 32 distinct banks, and the bias chunk they all
-// need is a broadcast.
+// rows of z (one contiguous block of 32 * E bf16) in shared memory with
+// coalesced 16-byte cp.async copies; for wide rows the next tile is
+// prefetched into L2, for narrow rows it is double-buffered.  Rows are padded
+// to a stride of 4 (mod 8) words, so the 32 lanes reading the same 16-byte
+// column chunk of their own rows hit 32 distinct banks and the per-expert
+// constants they need are broadcasts.
 //
-// Per token (s_e = fp32(z_e) + b_e, fp32 round-to-nearest-even):
-//   A. group maxima: element j of chunk c goes to group (c mod G/8)*8 + j;
-//      theta = the (K+1)st largest of the G group maxima.  K+1 distinct
-//      groups each hold an element >= theta, so theta <= tau_t.
-//   B. candidates: every e with s_e >= theta (a superset of the top-(K+1)
-//      set, ties included) is appended, in ascending e, to a per-lane list.
-//   C. exact selection: stable insertion of the candidates into a sorted
-//      (K+1)-list (a new candidate goes after equal scores, displaced
-//      entries shift down), so equal scores keep the lower index first.  A lane whose list overflows (many ties
-//      at theta) falls back to K+1 exact scans of its row.
+// Exact scores are s_e = fp32(z_e) + b_e (fp32, round to nearest even).  The
+// exact work is confined to a small candidate set found with packed bf16x2
+// arithmetic (two experts per instruction):
+//   A. lower bound: L_e = bf16(z_e + RD(b_e)) never exceeds the next bf16
+//      value above s_e, so the (K+1)st largest of G group maxima of L, moved
+//      down two bf16 steps, is <= tau_t (K+1 groups each hold an element at
+//      or above it).  Moving down two more steps gives the filter threshold.
+//   B. filter: U_e = bf16(z_e + RU(b_e)) >= threshold keeps every e with
+//      s_e >= tau_t (and a few more).  Per 8-expert chunk the passing experts
+//      form an 8-bit mask; chunks with a non-zero mask are listed per lane.
+//   C. exact selection: the listed experts, in ascending index, are inserted
+//      into a sorted (K+1)-list by their exact fp32 score; a new element goes
+//      after equal scores and displaced entries shift down, so ties keep the
+//      lower expert index first.  Any number of candidates (ties) is exact.
 // Loads are counted in per-warp shared counters for the warp's current
-// microbatch and flushed to global memory when the microbatch changes; each
-// warp owns a contiguous range of tiles, so flushes are rare.
+// microbatch and flushed to global memory when it changes; each warp owns a
+// contiguous range of tiles, so flushes are rare.
 #include "eqb_device.cuh"
 
 namespace eqb {
 
 namespace {
 
-constexpr int kCap = 32;   // candidate slots per token (power of two)
-constexpr int kNbuf = 2;   // tile buffers per warp
+constexpr int kEntries = 32;  // >= E/8 chunk entries per lane
 
 __host__ __device__ inline int row_stride_bytes(int E) {
-  int w = E / 2;                 // 32-bit words per row
-  return 4 * (w + ((4 - w) & 7));  // stride == 4 (mod 8) words
+  int w = E / 2;                     // 32-bit words per row
+  return 4 * (w + ((4 - w) & 7));    // stride == 4 (mod 8) words
 }
 
 __host__ __device__ inline int align16(int x) { return (x + 15) & ~15; }
 
-__host__ __device__ inline int warp_region_bytes(int E) {
-  return align16(kNbuf * 32 * row_stride_bytes(E) + kCap * 32 + 4 * E);
+__host__ __device__ inline int head_bytes(int E) { return align16(4 * E) + 2 * align16(2 * E); }
+
+__host__ __device__ inline int warp_region_bytes(int E, int nbuf) {
+  return align16(nbuf * 32 * row_stride_bytes(E) + kEntries * 32 * 2 + 4 * E);
 }
 
 template <int N>
@@ -80,8 +85,16 @@ __device__ __forceinline__ void insert_sorted(float (&v)[KP1], int (&id)[KP1], f
   }
 }
 
+// bf16 pattern `steps` representable values below x (toward -inf), clamped
+// at -inf.  Works on the order-preserving key.
+__device__ __forceinline__ uint32_t bf16_steps_down(uint32_t x, uint32_t steps) {
+  const uint32_t k = kappa16(x);
+  const uint32_t kmin = 0x0080u + steps;  // key of -max_finite is 0x0080
+  return k >= kmin ? kappa16_inv(k - steps) : 0xff80u;
+}
+
 template <int KP1, int G>
-__global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_per_warp) {
+__global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_per_warp, int nbuf) {
   extern __shared__ __align__(16) uint8_t smem[];
   const int E = a.E, K = a.K;
   const int nch = E >> 3;
@@ -91,16 +104,22 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
   const int nw = blockDim.x >> 5;
 
   float* bs = reinterpret_cast<float*>(smem);
-  const float4* bs4 = reinterpret_cast<const float4*>(smem);
-  uint8_t* wreg = smem + align16(4 * E) + wid * warp_region_bytes(E);
+  uint32_t* bdn = reinterpret_cast<uint32_t*>(smem + align16(4 * E));   // RD(b) packed pairs
+  uint32_t* bup = bdn + align16(2 * E) / 4;                              // RU(b) packed pairs
+  uint8_t* wreg = smem + head_bytes(E) + wid * warp_region_bytes(E, nbuf);
   uint8_t* tiles = wreg;
-  uint8_t* cand = wreg + kNbuf * tile_bytes;
-  int* wl = reinterpret_cast<int*>(cand + kCap * 32);
+  uint16_t* ent = reinterpret_cast<uint16_t*>(wreg + nbuf * tile_bytes);
+  int* wl = reinterpret_cast<int*>(wreg + nbuf * tile_bytes + kEntries * 32 * 2);
 
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
     const float v = a.b[e];
     bs[e] = v;
     if (!isfinite(v)) raise_flag(a.err, kErrNonfinite);
+  }
+  for (int q = threadIdx.x; q < E / 2; q += blockDim.x) {
+    const float b0 = a.b[2 * q], b1 = a.b[2 * q + 1];
+    bdn[q] = bf16_round_down(b0) | (bf16_round_down(b1) << 16);
+    bup[q] = bf16_round_up(b0) | (bf16_round_up(b1) << 16);
   }
   for (int e = lane; e < E; e += 32) wl[e] = 0;
   __syncthreads();
@@ -110,8 +129,10 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
   const int64_t tb = gw * tiles_per_warp;
   const int64_t te = min(tb + tiles_per_warp, ntiles);
   if (tb >= te) return;
+  const uint4* bdn4 = reinterpret_cast<const uint4*>(bdn);
+  const uint4* bup4 = reinterpret_cast<const uint4*>(bup);
 
-  // Issue the cp.async copies of one tile: row r, chunk `lane`.
+  // cp.async copies of one tile: row r, chunk `lane`.
   auto issue = [&](int64_t tile, int buf) {
     uint8_t* dst = tiles + buf * tile_bytes;
     const int64_t t0 = tile << 5;
@@ -122,6 +143,16 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
         const uint16_t* src = ok ? a.z + (t0 + r) * E + lane * 8 : a.z;
         cp_async16(dst + r * rs + lane * 16, src, ok ? 16 : 0);
       }
+    }
+  };
+  // Bring the given tile into L2 ahead of its cp.async copies.
+  auto prefetch = [&](int64_t tile) {
+    if (lane == 0 && tile < te) {
+      const int64_t t0 = tile << 5;
+      const int64_t rows = min((int64_t)32, a.T - t0);
+      const uint32_t bytes = static_cast<uint32_t>(rows * E * 2);
+      asm volatile("cp.async.bulk.prefetch.L2.global [%0], %1;" ::"l"(a.z + t0 * E), "r"(bytes)
+                   : "memory");
     }
   };
 
@@ -138,108 +169,103 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
     __syncwarp();
   };
 
-  issue(tb, 0);
-  cp_async_commit();
   int buf = 0;
-  for (int64_t tile = tb; tile < te; ++tile) {
-    if (tile + 1 < te) issue(tile + 1, buf ^ 1);
+  if (nbuf == 2) {
+    issue(tb, 0);
     cp_async_commit();
-    cp_async_wait<1>();
+  }
+  for (int64_t tile = tb; tile < te; ++tile) {
+    if (nbuf == 2) {
+      if (tile + 1 < te) issue(tile + 1, buf ^ 1);
+      cp_async_commit();
+      cp_async_wait<1>();
+    } else {
+      issue(tile, 0);
+      cp_async_commit();
+      prefetch(tile + 1);
+      cp_async_wait<0>();
+    }
     __syncwarp();
 
     const uint8_t* rowp = tiles + buf * tile_bytes + lane * rs;
     const int64_t t = (tile << 5) + lane;
     const bool valid = t < a.T;
 
-    // ---- A: group maxima and the lower bound theta <= tau_t
+    // ---- A: packed bf16 group maxima of the lower bounds L
     constexpr int U = G / 8;
-    float gm[G];
+    uint32_t gm2[G / 2];
 #pragma unroll
-    for (int g = 0; g < G; ++g) gm[g] = -INFINITY;
+    for (int g = 0; g < G / 2; ++g) gm2[g] = 0xff80ff80u;  // -inf, -inf
     for (int c0 = 0; c0 < nch; c0 += U) {
 #pragma unroll
       for (int u = 0; u < U; ++u) {
         const int c = c0 + u;
         if (c < nch) {
           const uint4 w = lds128(rowp + c * 16);
-          const float4 b0 = bs4[2 * c], b1 = bs4[2 * c + 1];
-          gm[u * 8 + 0] = fmax_nan(gm[u * 8 + 0], bf16_lo(w.x) + b0.x);
-          gm[u * 8 + 1] = fmax_nan(gm[u * 8 + 1], bf16_hi(w.x) + b0.y);
-          gm[u * 8 + 2] = fmax_nan(gm[u * 8 + 2], bf16_lo(w.y) + b0.z);
-          gm[u * 8 + 3] = fmax_nan(gm[u * 8 + 3], bf16_hi(w.y) + b0.w);
-          gm[u * 8 + 4] = fmax_nan(gm[u * 8 + 4], bf16_lo(w.z) + b1.x);
-          gm[u * 8 + 5] = fmax_nan(gm[u * 8 + 5], bf16_hi(w.z) + b1.y);
-          gm[u * 8 + 6] = fmax_nan(gm[u * 8 + 6], bf16_lo(w.w) + b1.z);
-          gm[u * 8 + 7] = fmax_nan(gm[u * 8 + 7], bf16_hi(w.w) + b1.w);
+          const uint4 bd = bdn4[c];
+          gm2[u * 4 + 0] = hmax2_nan_bf16(gm2[u * 4 + 0], hadd2_bf16(w.x, bd.x));
+          gm2[u * 4 + 1] = hmax2_nan_bf16(gm2[u * 4 + 1], hadd2_bf16(w.y, bd.y));
+          gm2[u * 4 + 2] = hmax2_nan_bf16(gm2[u * 4 + 2], hadd2_bf16(w.z, bd.z));
+          gm2[u * 4 + 3] = hmax2_nan_bf16(gm2[u * 4 + 3], hadd2_bf16(w.w, bd.w));
         }
       }
     }
+    float gm[G];
     bool has_nan = false;
 #pragma unroll
-    for (int g = 0; g < G; ++g) has_nan |= (gm[g] != gm[g]);
+    for (int g = 0; g < G / 2; ++g) {
+      gm[2 * g] = bf16_lo(gm2[g]);
+      gm[2 * g + 1] = bf16_hi(gm2[g]);
+      has_nan |= (gm[2 * g] != gm[2 * g]) || (gm[2 * g + 1] != gm[2 * g + 1]);
+    }
     if (has_nan && valid) raise_flag(a.err, kErrNonfinite);
     sort_desc<G>(gm);
     float theta = gm[0];
 #pragma unroll
     for (int g = 1; g < G; ++g) theta = (g == K) ? gm[g] : theta;
+    // Near zero, flushing of subnormal bf16 sums could move L by up to
+    // 2^-126; lowering theta below that range keeps the bound safe.
+    if (fabsf(theta) < 0x1p-124f) theta = -0x1p-124f;
+    const uint32_t thf = bf16_steps_down(__float_as_uint(theta) >> 16, 4u);
+    const uint32_t thf2 = thf | (thf << 16);
 
-    // ---- B: candidates s_e >= theta, ascending e
+    // ---- B: per-chunk masks of U >= threshold, chunks with a hit listed
     int cnt = 0;
     for (int c = 0; c < nch; ++c) {
       const uint4 w = lds128(rowp + c * 16);
-      const float4 b0 = bs4[2 * c], b1 = bs4[2 * c + 1];
-      float s[8];
-      s[0] = bf16_lo(w.x) + b0.x; s[1] = bf16_hi(w.x) + b0.y;
-      s[2] = bf16_lo(w.y) + b0.z; s[3] = bf16_hi(w.y) + b0.w;
-      s[4] = bf16_lo(w.z) + b1.x; s[5] = bf16_hi(w.z) + b1.y;
-      s[6] = bf16_lo(w.w) + b1.z; s[7] = bf16_hi(w.w) + b1.w;
-#pragma unroll
-      for (int j = 0; j < 8; ++j) {
-        if (s[j] >= theta) {
-          cand[((cnt & (kCap - 1)) << 5) | lane] = static_cast<uint8_t>(c * 8 + j);
-          ++cnt;
-        }
+      const uint4 bu = bup4[c];
+      const uint32_t r0 = hge2_bf16(hadd2_bf16(w.x, bu.x), thf2);
+      const uint32_t r1 = hge2_bf16(hadd2_bf16(w.y, bu.y), thf2);
+      const uint32_t r2 = hge2_bf16(hadd2_bf16(w.z, bu.z), thf2);
+      const uint32_t r3 = hge2_bf16(hadd2_bf16(w.w, bu.w), thf2);
+      // element 2q -> bit 2q (low half of r_q), element 2q+1 -> bit 16+2q
+      uint32_t y = r0 & 0x00010001u;
+      y |= r1 & 0x00040004u;
+      y |= r2 & 0x00100010u;
+      y |= r3 & 0x00400040u;
+      const uint32_t mask = (y | (y >> 15)) & 0xffu;
+      if (mask) {
+        ent[(cnt << 5) | lane] = static_cast<uint16_t>((c << 8) | mask);
+        ++cnt;
       }
     }
 
-    // ---- C: exact top-(K+1) among the candidates
+    // ---- C: exact top-(K+1) of the listed candidates
     float v[KP1];
     int id[KP1];
 #pragma unroll
     for (int j = 0; j < KP1; ++j) { v[j] = -INFINITY; id[j] = 0; }
-    const int n = min(__reduce_max_sync(kFull, cnt), kCap);
+    const int n = __reduce_max_sync(kFull, cnt);
     for (int i = 0; i < n; ++i) {
-      if (i < cnt) {
-        const int e = cand[(i << 5) | lane];
+      const uint32_t en = (i < cnt) ? ent[(i << 5) | lane] : 0u;
+      const int cbase = static_cast<int>(en >> 8) * 8;
+      uint32_t m = en & 0xffu;
+      while (m) {
+        const int j = __ffs(m) - 1;
+        m &= m - 1u;
+        const int e = cbase + j;
         const float s = bf16_bits_to_f32(*reinterpret_cast<const uint16_t*>(rowp + 2 * e)) + bs[e];
         insert_sorted<KP1>(v, id, s, e);
-      }
-    }
-    const bool overflow = cnt > kCap;
-    if (__any_sync(kFull, overflow)) {
-      if (overflow) {
-        // Exact fallback: K+1 scans, each taking the next element in the
-        // order (score descending, index ascending).
-        float pv = INFINITY;
-        int pi = -1;
-#pragma unroll 1
-        for (int k = 0; k < KP1; ++k) {
-          if (k <= K) {
-            float bv = -INFINITY;
-            int bi = 0;  // stays a valid index even if nothing qualifies (NaN rows)
-            bool found = false;
-            for (int e = 0; e < E; ++e) {
-              const float s = bf16_bits_to_f32(*reinterpret_cast<const uint16_t*>(rowp + 2 * e)) + bs[e];
-              const bool after = (s < pv) || (s == pv && e > pi);
-              if (after && (!found || s > bv)) { bv = s; bi = e; found = true; }
-            }
-#pragma unroll
-            for (int j = 0; j < KP1; ++j)
-              if (j == k) { v[j] = bv; id[j] = bi; }
-            pv = bv;
-            pi = bi;
-          }
-        }
       }
     }
     __syncwarp();
@@ -276,7 +302,7 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
       }
     }
     __syncwarp();
-    buf ^= 1;
+    if (nbuf == 2) buf ^= 1;
   }
   if (a.loads) flush_loads();
 }
@@ -286,8 +312,11 @@ int launch_route_kp1(const RouteArgs& a, cudaStream_t s) {
   constexpr int G = KP1 <= 16 ? 16 : 32;
   DeviceInfo di;
   if (int rc = device_info(&di)) return rc;
-  const int head = align16(4 * a.E);
-  const int wbytes = warp_region_bytes(a.E);
+  const int head = head_bytes(a.E);
+  // Wide rows: one tile buffer per warp (more resident warps) with an L2
+  // prefetch of the next tile; narrow rows: double buffering.
+  const int nbuf = a.E >= 128 ? 1 : 2;
+  const int wbytes = warp_region_bytes(a.E, nbuf);
   int nw = (di.max_smem_optin - head) / wbytes;
   if (nw > 16) nw = 16;
   if (nw < 1) return kErrUnsupported;
@@ -304,7 +333,7 @@ int launch_route_kp1(const RouteArgs& a, cudaStream_t s) {
   auto kern = route_kernel<KP1, G>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
     return kErrCuda;
-  kern<<<(unsigned)grid, nw * 32, smem, s>>>(a, tpw);
+  kern<<<(unsigned)grid, nw * 32, smem, s>>>(a, tpw, nbuf);
   return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
 }
 
