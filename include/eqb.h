@@ -33,7 +33,8 @@
  *    offsets[M] = T, non-decreasing (empty microbatches are allowed).
  *    The library reads them on the device; they are not checked on the host.
  *  - Supported sizes: 1 <= K, K + 1 <= 32, K < E, E a multiple of 8 with
- *    E <= 256, T < 2^31.  T = 0 is a valid no-op for the streaming calls.
+ *    E <= 256, T <= 2^31 - 2^24.  T = 0 is a valid no-op for the streaming
+ *    calls.
  *  - Device buffers of bf16 logits must be 16-byte aligned; fp32 gradient
  *    buffers 16-byte aligned.  Misaligned pointers give EQB_ERR_INVALID_ARG.
  */

@@ -49,7 +49,8 @@ inline eqb_status check_shape(int64_t T, int32_t E, int32_t K, bool need_k) {
   if (need_k && (K < 1 || K >= E)) return EQB_ERR_INVALID_ARG;
   if (E > 256 || (E % 8) != 0) return EQB_ERR_UNSUPPORTED;
   if (need_k && K + 1 > 32) return EQB_ERR_UNSUPPORTED;
-  if (T >= (int64_t(1) << 31)) return EQB_ERR_UNSUPPORTED;
+  // 32-bit token loop indices need headroom above T.
+  if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
   return EQB_OK;
 }
 

@@ -132,6 +132,10 @@ __device__ __forceinline__ uint32_t bf16_round_up(float x) {
   return (u & 0x80000000u) ? hi : hi + 1u;
 }
 
+__device__ __forceinline__ void prefetch_l2(const void* p) {
+  asm volatile("prefetch.global.L2 [%0];" ::"l"(p));
+}
+
 __device__ __forceinline__ void red_shared_add(uint32_t saddr, uint32_t v) {
   asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(saddr), "r"(v));
 }

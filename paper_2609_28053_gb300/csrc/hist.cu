@@ -68,47 +68,54 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
   }
   __syncthreads();
 
-  const int64_t tb = (int64_t)blockIdx.y * tokens_per_cta;
-  const int64_t te = min(tb + tokens_per_cta, a.T);
-  for (int64_t cb = tb; cb < te; cb += kFlushTokens) {
-    const int64_t ce = min(cb + kFlushTokens, te);
-    for (int64_t base_t = cb + (int64_t)wid * Lay::TPS; base_t < ce;
-         base_t += (int64_t)nw * Lay::TPS * kUnroll) {
+  // Token indices fit in 32 bits (T < 2^31 is checked on the host).
+  const int tb = static_cast<int>(min((int64_t)blockIdx.y * tokens_per_cta, a.T));
+  const int te = static_cast<int>(min((int64_t)tb + tokens_per_cta, a.T));
+  const int step = nw * Lay::TPS;  // tokens per warp round
+  const size_t zstride = static_cast<size_t>(step) * E;
+  const uint16_t* zlane = a.z + e0 + c * 8;
+
+  auto process = [&](const uint4& w4, float tv) {
+    const uint32_t zw[4] = {w4.x, w4.y, w4.z, w4.w};
+#pragma unroll
+    for (int p = 0; p < 4; ++p) {
+      const uint32_t m = pack_bf16x2_rn(tv - bf16_lo(zw[p]), tv - bf16_hi(zw[p]));
+      const uint32_t k = kappa2_internal(m);
+      const uint32_t row = base + 1024u * p;
+      if (PASS == 1) {
+        const uint32_t he = prmt(k, 0u, 0x4441u), ho = k >> 24;  // internal high bytes
+        const bool same = he == ho;
+        red_shared_add(row + 4u * he, same ? 0x10001u : 1u);
+        if (!same) red_shared_add(row + 4u * ho, 0x10000u);
+      } else {
+        const uint32_t d = (k ^ sel[p]) & 0xff00ff00u;
+        if ((d & 0x0000ff00u) == 0u) red_shared_add(row + 4u * (k & 0xffu), 1u);
+        if ((d & 0xff000000u) == 0u) red_shared_add(row + 4u * prmt(k, 0u, 0x4442u), 0x10000u);
+      }
+    }
+  };
+
+  for (int cb = tb; cb < te; cb += static_cast<int>(kFlushTokens)) {
+    const int ce = static_cast<int>(min((int64_t)cb + kFlushTokens, (int64_t)te));
+    int t = cb + wid * Lay::TPS + tok;
+    const uint16_t* zp = zlane + static_cast<size_t>(t) * E;
+    // full rounds of kUnroll tokens per lane, no guards
+    for (; t + (kUnroll - 1) * step < ce; t += kUnroll * step, zp += kUnroll * zstride) {
       uint4 w[kUnroll];
       float tt[kUnroll];
 #pragma unroll
       for (int u = 0; u < kUnroll; ++u) {
-        const int64_t t = base_t + (int64_t)u * nw * Lay::TPS + tok;
-        if (t < ce) {
-          w[u] = __ldcs(reinterpret_cast<const uint4*>(a.z + t * E + e0 + c * 8));
-          tt[u] = __ldg(a.tau + t);
-        } else {
-          w[u] = make_uint4(0, 0, 0, 0);
-          tt[u] = 0.f;
-        }
+        w[u] = __ldcs(reinterpret_cast<const uint4*>(zp + u * zstride));
+        tt[u] = __ldg(a.tau + t + u * step);
       }
+      // Pull the next round into L2 while this one is processed.
 #pragma unroll
-      for (int u = 0; u < kUnroll; ++u) {
-        const int64_t t = base_t + (int64_t)u * nw * Lay::TPS + tok;
-        if (t >= ce) continue;
-        const float tv = tt[u];
-        const uint32_t zw[4] = {w[u].x, w[u].y, w[u].z, w[u].w};
+      for (int u = 0; u < kUnroll; ++u)
+        if (t + (kUnroll + u) * step < ce) prefetch_l2(zp + (kUnroll + u) * zstride);
 #pragma unroll
-        for (int p = 0; p < 4; ++p) {
-          const uint32_t m = pack_bf16x2_rn(tv - bf16_lo(zw[p]), tv - bf16_hi(zw[p]));
-          const uint32_t k = kappa2_internal(m);
-          const uint32_t row = base + 1024u * p;
-          if (PASS == 1) {
-            red_shared_add(row + 4u * prmt(k, 0u, 0x4441u), 1u);        // even expert
-            red_shared_add(row + 4u * (k >> 24), 0x10000u);              // odd expert
-          } else {
-            const uint32_t d = (k ^ sel[p]) & 0xff00ff00u;
-            if ((d & 0x0000ff00u) == 0u) red_shared_add(row + 4u * (k & 0xffu), 1u);
-            if ((d & 0xff000000u) == 0u) red_shared_add(row + 4u * prmt(k, 0u, 0x4442u), 0x10000u);
-          }
-        }
-      }
+      for (int u = 0; u < kUnroll; ++u) process(w[u], tt[u]);
     }
+    for (; t < ce; t += step, zp += zstride) process(__ldcs(reinterpret_cast<const uint4*>(zp)), __ldg(a.tau + t));
     __syncthreads();
     // Flush: add every non-zero 16-bit counter to the global histogram.
     for (int i = threadIdx.x; i < Lay::kRows * 256; i += blockDim.x) {

@@ -21,8 +21,8 @@
 //      form an 8-bit mask; chunks with a non-zero mask are listed per lane.
 //   C. exact selection: the listed experts, in ascending index, are inserted
 //      into a sorted (K+1)-list by their exact fp32 score; a new element goes
-//      after equal scores and displaced entries shift down, so ties keep the
-//      lower expert index first.  Any number of candidates (ties) is exact.
+//      after equal scores, so ties keep the lower expert index first.  Any
+//      number of candidates (ties) is handled exactly.
 // Loads are counted in per-warp shared counters for the warp's current
 // microbatch and flushed to global memory when it changes; each warp owns a
 // contiguous range of tiles, so flushes are rare.
@@ -67,22 +67,22 @@ __device__ __forceinline__ void sort_desc(float (&a)[N]) {
 }
 
 // Insert (s, e) into the descending list (v, id).  Candidates arrive in
-// ascending e, so a new element goes after equal scores (strict compare);
-// once it has been placed, every later slot shifts down unconditionally.
+// ascending e, so the new element goes after equal scores: its slot is
+// p = #{j : v[j] >= s}; slots below p keep their entry, slot p takes the new
+// one, slots above p take their predecessor's.  Every slot is computed from
+// the old list, so there is no serial dependency between slots.
 template <int KP1>
 __device__ __forceinline__ void insert_sorted(float (&v)[KP1], int (&id)[KP1], float s, int e) {
-  bool moved = false;
+  bool ge[KP1];
 #pragma unroll
-  for (int j = 0; j < KP1; ++j) {
-    const bool gt = moved || s > v[j];
-    moved = gt;
-    const float tv = v[j];
-    const int ti = id[j];
-    v[j] = gt ? s : tv;
-    id[j] = gt ? e : ti;
-    s = gt ? tv : s;
-    e = gt ? ti : e;
+  for (int j = 0; j < KP1; ++j) ge[j] = v[j] >= s;
+#pragma unroll
+  for (int j = KP1 - 1; j >= 1; --j) {
+    v[j] = ge[j] ? v[j] : (ge[j - 1] ? s : v[j - 1]);
+    id[j] = ge[j] ? id[j] : (ge[j - 1] ? e : id[j - 1]);
   }
+  v[0] = ge[0] ? v[0] : s;
+  id[0] = ge[0] ? id[0] : e;
 }
 
 // bf16 pattern `steps` representable values below x (toward -inf), clamped
@@ -255,15 +255,22 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
     int id[KP1];
 #pragma unroll
     for (int j = 0; j < KP1; ++j) { v[j] = -INFINITY; id[j] = 0; }
-    const int n = __reduce_max_sync(kFull, cnt);
-    for (int i = 0; i < n; ++i) {
-      const uint32_t en = (i < cnt) ? ent[(i << 5) | lane] : 0u;
-      const int cbase = static_cast<int>(en >> 8) * 8;
-      uint32_t m = en & 0xffu;
-      while (m) {
-        const int j = __ffs(m) - 1;
+    // One candidate per lane per iteration: a lane whose current chunk mask
+    // is used up loads its next entry, so the warp runs for the largest
+    // candidate count of its lanes.
+    int ei = 0, cbase = 0;
+    uint32_t m = 0u;
+    for (;;) {
+      if (m == 0u && ei < cnt) {
+        const uint32_t en = ent[(ei << 5) | lane];
+        cbase = static_cast<int>(en >> 8) * 8;
+        m = en & 0xffu;
+        ++ei;
+      }
+      if (!__any_sync(kFull, m != 0u)) break;
+      if (m != 0u) {
+        const int e = cbase + __ffs(m) - 1;
         m &= m - 1u;
-        const int e = cbase + j;
         const float s = bf16_bits_to_f32(*reinterpret_cast<const uint16_t*>(rowp + 2 * e)) + bs[e];
         insert_sorted<KP1>(v, id, s, e);
       }
