@@ -153,6 +153,23 @@ eqb_status lei_inject_grad(float *grad_s, const int32_t *loads,
                            const int64_t *mb_offsets, int32_t M, int64_t T,
                            int32_t E, int32_t K, float eta, float c, void *stream);
 
+/* Router logits, Sec. 2 (Eq. 1: z_t = W_r x_t):
+ *   z[t, e] = bf16_rne(sum_k x[t, k] * W_r[e, k]),
+ * bf16 inputs, fp32 accumulation on the tensor cores (tcgen05, accumulators
+ * in tensor memory).  The accumulation order is the hardware's, so an entry
+ * can differ from the exactly rounded value by one bf16 ulp plus the fp32
+ * accumulation error.
+ *   x        device bf16 [T, d] row-major, 16-byte aligned     (in)
+ *   W_r      device bf16 [E, d] row-major, 16-byte aligned     (in)
+ *   z        device bf16 [T, E] row-major, 16-byte aligned     (out)
+ *   err_flag device int32 (nullable): EQB_ERR_CUDA if the kernel's pipeline
+ *            stalled and it gave up waiting (no result is then valid).
+ * Supported: d a positive multiple of 64, E a multiple of 16 with
+ * 16 <= E <= 256, 0 <= T <= 2^31 - 2^24.  Uses all tensor memory of each SM
+ * it runs on, one block per SM. */
+eqb_status eqb_router_logits(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t T, int32_t d,
+                             int32_t E, eqb_bf16 *z, int32_t *err_flag, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -16,6 +16,7 @@ Every wrapper cites the passage of arXiv 2609.28053 it follows:
   :func:`select_lo`        -- Algorithm 1, steps 3, 5 and 6.
 * :func:`bias_update`      -- Eq. (2) centering.
 * :func:`lei`              -- Sec. 4, Eq. (LEI) with Eq. (norm).
+* :func:`router_logits`    -- Sec. 2, z_t = W_r x_t, dot products in fp64.
 """
 from __future__ import annotations
 
@@ -68,6 +69,7 @@ def _load():
                 "oracle_select_lo": [P, i32, P, P, P],
                 "oracle_bias_update": [P, i32, P],
                 "oracle_lei": [P, P, P, i32, i64, i32, i32, f32, f32, P, P],
+                "oracle_router_logits": [P, P, i64, i32, i32, P, i64, P, P],
             }
             for name, args in sig.items():
                 fn = getattr(lib, name)
@@ -247,6 +249,21 @@ def lei(g, loads, offsets, K, eta, c):
                             float(eta), float(c), _ptr(g_out), _ptr(a))
     _check(rc, "oracle_lei")
     return g_out, a
+
+
+def router_logits(x_bits, W_bits, rows):
+    """Sec. 2: z_t = W_r x_t for the listed rows, in fp64.  Returns
+    (z float64 [n,E], sum of |products| float64 [n,E])."""
+    x_bits = _c(x_bits, np.uint16)
+    W_bits = _c(W_bits, np.uint16)
+    T, d = x_bits.shape
+    E = W_bits.shape[0]
+    rows = _c(rows, np.int64)
+    out = np.zeros((len(rows), E), np.float64)
+    ab = np.zeros((len(rows), E), np.float64)
+    _check(_load().oracle_router_logits(_ptr(x_bits), _ptr(W_bits), T, d, E, _ptr(rows), len(rows),
+                                        _ptr(out), _ptr(ab)), "oracle_router_logits")
+    return out, ab
 
 
 def eqb_step(z_bits, b, K, offsets=None):

@@ -18,6 +18,7 @@
  *                reaching the rank).
  *   bias update  Eq. (2) centering b = b_hat - mean(b_hat).
  *   LEI          Sec. 4, Eq. (LEI) and Eq. (norm).
+ *   router       Sec. 2: z_t = W_r x_t, the dot products in fp64.
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - scores s = fp32(z) + b in fp32 round-to-nearest-even; tau is fp32;
@@ -332,5 +333,30 @@ int oracle_lei(const float *g, const int32_t *loads, const int64_t *off,
           g_out[t * E + e] = (float)((double)g[t * E + e] + a[e]);
   }
   free(a);
+  return ORACLE_OK;
+}
+
+/* ---- router projection: Sec. 2, z_t = W_r x_t -------------------------- */
+
+/* For each listed row t: out[i, e] = sum_k x[t, k] * W[e, k] in fp64 (each
+ * product of two bf16 values is exact in fp64) and abs_out[i, e] =
+ * sum_k |x[t, k] * W[e, k]| (the scale of the accumulation error). */
+int oracle_router_logits(const uint16_t *x, const uint16_t *W, int64_t T, int32_t d, int32_t E,
+                         const int64_t *rows, int64_t n_rows, double *out, double *abs_out) {
+  if (T < 0 || d < 1 || E < 1) return ORACLE_ERR_ARG;
+  for (int64_t i = 0; i < n_rows; ++i) {
+    int64_t t = rows[i];
+    if (t < 0 || t >= T) return ORACLE_ERR_ARG;
+    for (int32_t e = 0; e < E; ++e) {
+      double acc = 0.0, acc_abs = 0.0;
+      for (int32_t k = 0; k < d; ++k) {
+        double p = (double)bf16_bits_to_f32(x[t * d + k]) * (double)bf16_bits_to_f32(W[(int64_t)e * d + k]);
+        acc += p;
+        acc_abs += fabs(p);
+      }
+      out[i * E + e] = acc;
+      if (abs_out) abs_out[i * E + e] = acc_abs;
+    }
+  }
   return ORACLE_OK;
 }

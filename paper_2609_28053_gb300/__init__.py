@@ -15,6 +15,9 @@ The routing-balance step of one MoE layer, in the paper's order:
     eqb_select_quantile   Algorithm 1 steps 5-6 (pass 2): exact quantile
     eqb_bias_update       Eq. (2): centred bias for the next step
     lei_inject_grad       Sec. 4: Eq. (LEI) with Eq. (norm)
+
+and, for layers whose logits are produced here, eqb_router_logits (Sec. 2,
+z_t = W_r x_t) on the tensor cores.
 """
 from __future__ import annotations
 
@@ -27,7 +30,7 @@ from ._lib import STATUS, EqbError, load
 __all__ = [
     "EqbError", "STATUS", "load", "eqb_target_rank", "eqb_route_topk", "eqb_margin_hist_pass1",
     "eqb_margin_hist_pass2", "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad",
-    "EqbWorkspace", "eqb_layer_forward",
+    "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits",
 ]
 
 
@@ -136,6 +139,22 @@ def lei_inject_grad(grad_s, loads, mb_offsets, K, eta, c, stream=None):
     _need(loads, torch.int32, "loads", (M, E))
     _check(load().lei_inject_grad(_p(grad_s), _p(loads), _p(mb_offsets), M, T, E, K, float(eta),
                                   float(c), _stream(stream)), "lei_inject_grad")
+
+
+def eqb_router_logits(x, W_r, z=None, err_flag=None, stream=None):
+    """Router logits z = bf16(x W_r^T), fp32 accumulation on the tensor cores.
+    x bf16 [T,d], W_r bf16 [E,d]; returns z bf16 [T,E]."""
+    T, d = x.shape
+    E = W_r.shape[0]
+    _need(x, torch.bfloat16, "x")
+    _need(W_r, torch.bfloat16, "W_r", (E, d))
+    if z is None:
+        z = torch.empty((T, E), dtype=torch.bfloat16, device=x.device)
+    _need(z, torch.bfloat16, "z", (T, E))
+    _need(err_flag, torch.int32, "err_flag")
+    _check(load().eqb_router_logits(_p(x), _p(W_r), T, d, E, _p(z), _p(err_flag), _stream(stream)),
+           "eqb_router_logits")
+    return z
 
 
 class EqbWorkspace:

@@ -15,7 +15,7 @@ LIB_PATH = os.path.join(HERE, "libeqb.so")
 EXPORTS = (
     "eqb_status_string", "eqb_version", "eqb_target_rank", "eqb_route_topk",
     "eqb_margin_hist_pass1", "eqb_margin_hist_pass2", "eqb_select_quantile",
-    "eqb_bias_update", "lei_inject_grad",
+    "eqb_bias_update", "lei_inject_grad", "eqb_router_logits",
 )
 
 STATUS = {0: "EQB_OK", 1: "EQB_ERR_INVALID_ARG", 2: "EQB_ERR_UNSUPPORTED", 3: "EQB_ERR_CUDA",
@@ -50,6 +50,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
             "eqb_select_quantile": [P, i32, i32, i64, P, P, P, P, P],
             "eqb_bias_update": [P, i32, P, P],
             "lei_inject_grad": [P, P, P, i32, i64, i32, i32, f32, f32, P],
+            "eqb_router_logits": [P, P, i64, i32, i32, P, P, P],
         }
         for name, args in sigs.items():
             fn = getattr(lib, name)

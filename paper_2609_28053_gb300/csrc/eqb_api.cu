@@ -155,4 +155,16 @@ eqb_status lei_inject_grad(float* grad_s, const int32_t* loads, const int64_t* m
   return to_status(eqb::launch_lei(a, as_stream(stream)));
 }
 
+eqb_status eqb_router_logits(const eqb_bf16* x, const eqb_bf16* W_r, int64_t T, int32_t d, int32_t E,
+                             eqb_bf16* z, int32_t* err_flag, void* stream) {
+  if (T < 0 || d < 1 || E < 1) return EQB_ERR_INVALID_ARG;
+  if ((d % 64) != 0 || (E % 16) != 0 || E > 256) return EQB_ERR_UNSUPPORTED;
+  if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
+  if (!x || !W_r || !z) return EQB_ERR_INVALID_ARG;
+  if (!aligned(x, 16) || !aligned(W_r, 16) || !aligned(z, 16) || !aligned(err_flag, 4))
+    return EQB_ERR_INVALID_ARG;
+  if (T == 0) return EQB_OK;
+  return to_status(eqb::launch_router_gemm(x, W_r, T, d, E, z, err_flag, as_stream(stream)));
+}
+
 }  // extern "C"

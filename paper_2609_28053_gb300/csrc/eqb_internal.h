@@ -64,5 +64,7 @@ int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, i
                   uint16_t* q_hat, int32_t* err, cudaStream_t s);
 int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t s);
 int launch_lei(const LeiArgs& a, cudaStream_t s);
+int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, uint16_t* z,
+                       int32_t* err, cudaStream_t s);
 
 }  // namespace eqb

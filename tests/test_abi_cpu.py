@@ -109,3 +109,14 @@ def test_binding_fails_loudly_without_library(tmp_path):
     from paper_2609_28053_gb300 import _lib
     with pytest.raises(RuntimeError, match="no CPU fallback"):
         _lib.load(str(tmp_path / "missing.so"))
+
+
+def test_router_logits_rejects(lib):
+    f = lib.eqb_router_logits
+    assert f(FAKE, FAKE, 10, 4096, 8, FAKE, NULL, NULL) == UNSUPPORTED     # E not a multiple of 16
+    assert f(FAKE, FAKE, 10, 4000, 128, FAKE, NULL, NULL) == UNSUPPORTED   # d not a multiple of 64
+    assert f(FAKE, FAKE, 10, 4096, 272, FAKE, NULL, NULL) == UNSUPPORTED   # E > 256
+    assert f(NULL, FAKE, 10, 4096, 128, FAKE, NULL, NULL) == INVALID
+    assert f(FAKE, FAKE, -1, 4096, 128, FAKE, NULL, NULL) == INVALID
+    assert f(MISALIGNED, FAKE, 10, 4096, 128, FAKE, NULL, NULL) == INVALID
+    assert f(FAKE, FAKE, 0, 4096, 128, FAKE, NULL, NULL) == 0

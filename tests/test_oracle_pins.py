@@ -316,3 +316,24 @@ def test_target_rank():
     assert oracle.target_rank(2097152, 256, 8) == 65536
     assert oracle.target_rank(1048576, 128, 8) == 65536
     assert oracle.target_rank(10, 8, 3) == 4  # ceil(30/8)
+
+
+# ---------------------------------------------------------------- router projection
+
+def test_router_logits_matches_float64_matmul_and_one_hot():
+    """Sec. 2: z_t = W_r x_t.  Pinned against numpy's float64 matmul (a
+    library routine) and the one-hot closed form (x = e_k picks column k)."""
+    rng = np.random.default_rng(21)
+    T, d, E = 37, 192, 24
+    x = brute.bf16_bits_from_f32(rng.standard_normal((T, d)).astype(np.float32))
+    W = brute.bf16_bits_from_f32((rng.standard_normal((E, d)) / np.sqrt(d)).astype(np.float32))
+    rows = np.arange(T)
+    z, ab = oracle.router_logits(x, W, rows)
+    xf = brute.f32_from_bf16_bits(x).astype(np.float64)
+    Wf = brute.f32_from_bf16_bits(W).astype(np.float64)
+    assert np.allclose(z, xf @ Wf.T, rtol=1e-12, atol=1e-12)
+    assert np.allclose(ab, np.abs(xf) @ np.abs(Wf).T, rtol=1e-12, atol=1e-12)
+    onehot = np.zeros((d, d), np.float32)
+    np.fill_diagonal(onehot, 1.0)
+    zo, _ = oracle.router_logits(brute.bf16_bits_from_f32(onehot), W, np.arange(0, d, 7))
+    assert np.array_equal(zo, Wf[:, ::7].T)
