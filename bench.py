@@ -108,24 +108,56 @@ class ClockSampler:
 
 
 class Step:
-    """Device buffers and the launch sequence of one routing-balance step."""
+    """Device buffers and the launch sequence of one routing-balance step.
 
-    def __init__(self, T, E, K, M, dev, seed_shift=0):
+    workload 'global': logits resident in HBM (T=2,097,152, E=256, K=8).
+    workload 'router': the router projection on the tensor cores first
+    (x [T,4096] bf16, W_r [128,4096]), then the same path on its logits; the
+    bias produced by a step is the next step's bias (Eq. 2)."""
+
+    def __init__(self, workload, T, dev, seed_shift=0):
         import paper_2609_28053_gb300 as eqb
+        from eqb_workloads import make_router_inputs
         self.eqb = eqb
-        self.T, self.E, self.K, self.M = T, E, K, M
-        self.z = make_logits("global", T=T, seed=SHAPES["global"].seed + seed_shift, device=str(dev))
-        self.b = make_bias("global", device=str(dev))
-        self.g = make_grad("global", T=T, device=str(dev))
-        self.off = torch.from_numpy(even_offsets(T, M)).to(dev)
+        self.workload = workload
+        sh = SHAPES[workload]
+        self.T, self.E, self.K = T, sh.E, sh.K
+        self.M = max(1, T // (sh.T // sh.M))
+        E = self.E
+        if workload == "router":
+            self.x, self.W = make_router_inputs(T=T, step=seed_shift, device=str(dev))
+            self.d = self.x.shape[1]
+            self.z = torch.empty((T, E), dtype=torch.bfloat16, device=dev)
+            self.b = torch.zeros(E, dtype=torch.float32, device=dev)
+        else:
+            self.z = make_logits(workload, T=T, seed=sh.seed + seed_shift, device=str(dev))
+            self.b = make_bias(workload, device=str(dev))
+        self.g = make_grad(workload, T=T, device=str(dev))
+        self.off = torch.from_numpy(even_offsets(T, self.M)).to(dev)
         self.ws = eqb.EqbWorkspace(E, device=dev)
-        self.idx = torch.empty((T, K), dtype=torch.int32, device=dev)
+        self.idx = torch.empty((T, self.K), dtype=torch.int32, device=dev)
         self.tau = torch.empty(T, dtype=torch.float32, device=dev)
-        self.loads = torch.zeros((M, E), dtype=torch.int32, device=dev)
+        self.loads = torch.zeros((self.M, E), dtype=torch.int32, device=dev)
         self.b_next = torch.empty(E, dtype=torch.float32, device=dev)
         self.r_global = None
-        self.names = ["route_topk", "margin_hist_pass1", "select_pass1", "margin_hist_pass2",
-                      "select_pass2", "bias_update", "lei_inject_grad"]
+        self.off_h = even_offsets(T, self.M)
+        self.workspace = torch.zeros(eqb.eqb_layer_workspace_bytes(E), dtype=torch.uint8, device=dev)
+        self.names = (["router_logits"] if workload == "router" else []) + [
+            "route_topk", "margin_hist_pass1", "select_pass1", "margin_hist_pass2",
+            "select_pass2", "bias_update", "lei_inject_grad"]
+
+    def run_step(self, stream):
+        """One step through the one-call entry point eqb_layer_step: routing,
+        both histogram passes, selections, the bias update and LEI."""
+        eqb = self.eqb
+        if self.workload == "router":
+            eqb.eqb_router_logits(self.x, self.W, self.z, self.ws.err, stream)
+        eqb.eqb_layer_step(self.z, self.b, self.K, self.off, self.loads, self.b_next, self.workspace,
+                           tau=self.tau, topk_idx=self.idx, grad_s=self.g, eta=ETA, c=C_NORM,
+                           mb_offsets_host=self.off_h, r=self.r_global or 0, err_flag=self.ws.err,
+                           stream=stream)
+        if self.workload == "router":
+            self.b.copy_(self.b_next)  # b^(q+1) routes step q+1
 
     def run(self, stream, world=1, events=None, z=None, g=None):
         """Enqueue one step.  `events` (optional) is a list of (start, end)
@@ -134,6 +166,7 @@ class Step:
         z = self.z if z is None else z
         g = self.g if g is None else g
         r = self.r_global or eqb.eqb_target_rank(self.T * world, self.E, self.K)
+        i0 = 0
 
         def rec(i, fn):
             if events is not None:
@@ -146,29 +179,46 @@ class Step:
         ws.hist_lo.zero_()
         ws.err.zero_()
         self.loads.zero_()
-        rec(0, lambda: eqb.eqb_route_topk(z, self.b, self.K, self.off, self.idx, self.tau, self.loads,
-                                          None, ws.err, stream))
-        rec(1, lambda: eqb.eqb_margin_hist_pass1(z, self.tau, ws.hist_hi, ws.err, stream))
+        if self.workload == "router":
+            rec(0, lambda: eqb.eqb_router_logits(self.x, self.W, z, ws.err, stream))
+            i0 = 1
+        rec(i0 + 0, lambda: eqb.eqb_route_topk(z, self.b, self.K, self.off, self.idx, self.tau,
+                                               self.loads, None, ws.err, stream))
+        rec(i0 + 1, lambda: eqb.eqb_margin_hist_pass1(z, self.tau, ws.hist_hi, ws.err, stream))
         if world > 1:
             torch.distributed.all_reduce(ws.hist_hi)
-        rec(2, lambda: eqb.eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream))
-        rec(3, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
+        rec(i0 + 2, lambda: eqb.eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream))
+        rec(i0 + 3, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
         if world > 1:
             torch.distributed.all_reduce(ws.hist_lo)
-        rec(4, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err, stream))
-        rec(5, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
-        rec(6, lambda: eqb.lei_inject_grad(g, self.loads, self.off, self.K, ETA, C_NORM, stream))
+        rec(i0 + 4, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err,
+                                                    stream))
+        rec(i0 + 5, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
+        rec(i0 + 6, lambda: eqb.lei_inject_grad(g, self.loads, self.off, self.K, ETA, C_NORM, stream))
+        if self.workload == "router":
+            self.b.copy_(self.b_next)  # b^(q+1) routes step q+1
+
+    def launches_per_step(self):
+        """Kernels of this library launched by one timed step (memsets and
+        torch copies excluded): routing, two histogram passes, two
+        selections, the bias update and LEI (+ the router GEMM)."""
+        return 7 + (1 if self.workload == "router" else 0)
 
     def algorithmic_bytes(self):
         """Bytes the two-pass method must move per step (see the design notes):
         pass 1 reads z (2TE) and writes idx (4TK) and tau (4T); pass 2 reads z
-        (2TE) and tau (4T); LEI reads and writes grad (8TE).  Per kernel:"""
+        (2TE) and tau (4T); LEI reads and writes grad (8TE); the router
+        projection reads x (2Td) and W_r (2Ed) and writes z (2TE).  Per kernel:"""
         T, E, K = self.T, self.E, self.K
-        return {"route_topk": 2 * T * E + 4 * T * K + 4 * T,
-                "margin_hist_pass1": 2 * T * E + 4 * T,
-                "margin_hist_pass2": 2 * T * E + 4 * T,
-                "lei_inject_grad": 8 * T * E,
-                "path": 12 * T * E + 8 * T + 4 * T * K}
+        d = {"route_topk": 2 * T * E + 4 * T * K + 4 * T,
+             "margin_hist_pass1": 2 * T * E + 4 * T,
+             "margin_hist_pass2": 2 * T * E + 4 * T,
+             "lei_inject_grad": 8 * T * E,
+             "path": 12 * T * E + 8 * T + 4 * T * K}
+        if self.workload == "router":
+            d["router_logits"] = 2 * T * self.d + 2 * E * self.d + 2 * T * E
+            d["path"] += d["router_logits"]
+        return d
 
 
 def cpu_oracle_sample(z_dev, b_dev, g_dev, K, n_tokens, M_per):
@@ -184,6 +234,23 @@ def cpu_oracle_sample(z_dev, b_dev, g_dev, K, n_tokens, M_per):
     oracle.build()
     t0 = time.perf_counter()
     st = oracle.eqb_step(zb, bh, K, off)
+    oracle.lei(gh, st["loads"], off, K, ETA, C_NORM)
+    return time.perf_counter() - t0, n_tokens
+
+
+def cpu_oracle_router_sample(x_dev, W_dev, g_dev, K, n_tokens):
+    """The oracle on the router workload's first n_tokens: the projection
+    z_t = W_r x_t in fp64 rounded to bf16, then the routing-balance step."""
+    import oracle
+    from eqb_workloads import bits
+    xb, Wb = bits(x_dev[:n_tokens]), bits(W_dev)
+    gh = g_dev[:n_tokens].cpu().numpy()
+    off = even_offsets(n_tokens, 1)
+    oracle.build()
+    t0 = time.perf_counter()
+    z64, _ = oracle.router_logits(xb, Wb, np.arange(n_tokens))
+    zb = torch.from_numpy(z64.astype(np.float32)).to(torch.bfloat16).view(torch.int16).numpy().view(np.uint16)
+    st = oracle.eqb_step(zb, np.zeros(Wb.shape[0], np.float32), K, off)
     oracle.lei(gh, st["loads"], off, K, ETA, C_NORM)
     return time.perf_counter() - t0, n_tokens
 
@@ -222,7 +289,8 @@ def main():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--tokens", type=int, default=SHAPES["global"].T)
+    ap.add_argument("--workload", default="global", choices=["global", "router"])
+    ap.add_argument("--tokens", type=int, default=None)
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-sample-tokens", type=int, default=131072)
     ap.add_argument("--ref-sample-tokens", type=int, default=32768)
@@ -239,9 +307,10 @@ def main():
         torch.distributed.init_process_group("nccl")
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
-    sh = SHAPES["global"]
-    T, E, K, M = args.tokens, sh.E, sh.K, max(1, args.tokens // 32768)
-    step = Step(T, E, K, M, dev, seed_shift=rank)
+    sh = SHAPES[args.workload]
+    T = args.tokens or sh.T
+    step = Step(args.workload, T, dev, seed_shift=rank)
+    E, K, M = step.E, step.K, step.M
     step.r_global = step.eqb.eqb_target_rank(T * world, E, K)
     stream = torch.cuda.current_stream()
 
@@ -250,23 +319,29 @@ def main():
             torch.distributed.barrier()
         torch.cuda.synchronize()
 
+    one_call = world == 1  # the one-call step keeps its histograms local
+
+    def do_step():
+        if one_call:
+            step.run_step(stream)
+        else:
+            step.run(stream, world)
+
     for _ in range(args.warmup):
-        step.run(stream, world)
+        do_step()
     barrier()
     err = step.ws.err.item()
     if err:
         raise RuntimeError(f"device flagged {step.eqb.STATUS.get(err, err)}")
 
-    nk = len(step.names)
-    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-            for _ in range(nk)] for _ in range(args.steps)]
     t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
     clocks = ClockSampler(local)
     barrier()
     clocks.start()
+    time.sleep(0.3)  # let the sampler start before the timed region
     t_start.record(stream)
-    for s in range(args.steps):
-        step.run(stream, world, events=evs[s])
+    for s_ in range(args.steps):
+        do_step()
     t_end.record(stream)
     barrier()
     clk = clocks.stop()
@@ -278,9 +353,19 @@ def main():
     ms_per_step = ms / args.steps
     value = world * T / (ms_per_step / 1e3)
 
+    # Per-kernel durations: the same work issued kernel by kernel on one
+    # stream, each launch bracketed by CUDA events, in its own timed loop.
+    nk = len(step.names)
+    ksteps = max(3, min(args.steps, 20))
+    evs = [[(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            for _ in range(nk)] for _ in range(ksteps)]
+    for s_ in range(ksteps):
+        step.run(stream, world, events=evs[s_])
+    barrier()
     per_kernel = {}
     for i, name in enumerate(step.names):
-        per_kernel[name] = statistics.mean(evs[s][i][0].elapsed_time(evs[s][i][1]) for s in range(args.steps))
+        per_kernel[name] = statistics.mean(evs[s_][i][0].elapsed_time(evs[s_][i][1]) for s_ in range(ksteps))
+    seq_ms = sum(per_kernel.values())
     alg = step.algorithmic_bytes()
     peak, peak_kind = measured_peaks()
     dom = max(per_kernel, key=per_kernel.get)
@@ -301,24 +386,26 @@ def main():
                    **({"GB/s": round(alg[k] / (v * 1e-3) / 1e9, 1), "frac": round(alg[k] / (v * 1e-3) / 1e9 / peak, 4)}
                       if k in alg else {})} for k, v in per_kernel.items()}
 
-    # ---- end to end through the public API with pinned host buffers
+    # ---- end to end through the public API with pinned host buffers: the
+    # step's inputs (logits, or activations for the router workload, and the
+    # score gradients) are copied in and its results (gradients, next bias,
+    # loads) copied out inside the timed region.
     e2e = None
     if args.e2e_steps > 0:
-        z_h = step.z.cpu().pin_memory()
+        src = step.x if args.workload == "router" else step.z
+        src_h = src.cpu().pin_memory()
         g_h = step.g.cpu().pin_memory()
         g_out = torch.empty_like(g_h).pin_memory()
         bn_out = torch.empty(E, dtype=torch.float32).pin_memory()
         ld_out = torch.empty((M, E), dtype=torch.int32).pin_memory()
-        z_d = torch.empty_like(step.z)
-        g_d = torch.empty_like(step.g)
-        h2d = z_h.numel() * 2 + g_h.numel() * 4
+        h2d = src_h.numel() * src_h.element_size() + g_h.numel() * 4
         d2h = g_out.numel() * 4 + bn_out.numel() * 4 + ld_out.numel() * 4
 
         def e2e_step():
-            z_d.copy_(z_h, non_blocking=True)
-            g_d.copy_(g_h, non_blocking=True)
-            step.run(stream, world, z=z_d, g=g_d)
-            g_out.copy_(g_d, non_blocking=True)
+            src.copy_(src_h, non_blocking=True)
+            step.g.copy_(g_h, non_blocking=True)
+            do_step()
+            g_out.copy_(step.g, non_blocking=True)
             bn_out.copy_(step.b_next, non_blocking=True)
             ld_out.copy_(step.loads, non_blocking=True)
 
@@ -340,26 +427,38 @@ def main():
 
     cpu_base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        n = min(args.cpu_sample_tokens, T)
-        secs, toks = cpu_oracle_sample(step.z, step.b, step.g, K, n, 32768)
+        n = min(args.cpu_sample_tokens if args.workload == "global" else 8192, T)
+        if args.workload == "router":
+            secs, toks = cpu_oracle_router_sample(step.x, step.W, step.g, K, n)
+            what = (f"first {n} tokens: router projection in fp64, routing, exact quantile of all "
+                    f"{E} experts by full sort, bias update, LEI")
+        else:
+            secs, toks = cpu_oracle_sample(step.z, step.b, step.g, K, n, 32768)
+            what = (f"first {n} tokens of the workload ({max(1, n // 32768)} microbatches): routing, "
+                    f"exact quantile of all {E} experts by full sort, bias update, LEI")
         cpu_base = {"value": toks / secs, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                    "sample": f"first {n} tokens of the workload ({max(1, n // 32768)} microbatches): "
-                              f"routing, exact quantile of all {E} experts by full sort, bias update, LEI",
-                    "seconds": secs, "host_cores_available": len(os.sched_getaffinity(0))}
+                    "sample": what, "seconds": secs,
+                    "host_cores_available": len(os.sched_getaffinity(0))}
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
                 "data": "synthetic",
-                "config": {"workload": f"global: T={T} E={E} K={K} M={M} per GPU, bf16 logits",
+                "config": {"workload": (f"global: T={T} E={E} K={K} M={M} per GPU, bf16 logits"
+                                        if args.workload == "global" else
+                                        f"router: x [{T},{step.d}] bf16, W_r [{E},{step.d}], "
+                                        f"E={E} K={K} M={M} per GPU, bias iterated"),
                            "T": T, "E": E, "K": K, "M": M, "eta": ETA, "c": C_NORM,
-                           "l2": "inputs larger than L2 (z 1 GiB, grad 2 GiB); no flush",
+                           "l2": "inputs larger than L2 (at least 1 GiB each); no flush",
                            "parallelism": f"dp{world}"},
-                "gpu_launches": nk * args.steps,
+                "gpu_launches": step.launches_per_step() * args.steps,
+                "schedule": ("one eqb_layer_step call per step" if one_call
+                             else "per-pass calls, histograms all-reduced"),
                 "roofline": roofline,
                 "path": {"algorithmic_bytes": alg["path"], "GB/s": path_gbs, "frac": path_gbs / peak},
                 "kernels": kernels,
+                "kernels_sequential_ms": seq_ms,
                 "clocks": clk, "e2e": e2e, "cpu_baseline": cpu_base,
                 "elements_per_s": value * E}
         print(json.dumps(line), flush=True)

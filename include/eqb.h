@@ -41,6 +41,7 @@
 #ifndef EQB_H
 #define EQB_H
 
+#include <stddef.h>
 #include <stdint.h>
 
 #ifdef __cplusplus
@@ -152,6 +153,33 @@ eqb_status eqb_bias_update(const eqb_bf16 *q_hat, int32_t E, float *b_next,
 eqb_status lei_inject_grad(float *grad_s, const int32_t *loads,
                            const int64_t *mb_offsets, int32_t M, int64_t T,
                            int32_t E, int32_t K, float eta, float c, void *stream);
+
+/* Bytes of device workspace eqb_layer_step needs for E experts (the two
+ * [E,256] histograms, u, rho and q_hat, each 256-byte aligned). */
+size_t eqb_layer_workspace_bytes(int32_t E);
+
+/* One layer's whole routing-balance step in one call, in the paper's order:
+ * routing (Sec. 2), Algorithm 1's coarse pass, selection, fine pass,
+ * selection, the Eq. (2) bias update, then Load-Error Injection (Sec. 4,
+ * Eqs. LEI and norm) on grad_s when grad_s is given.  Results are identical
+ * to the individual calls above.
+ *   z, b, mb_offsets, M, topk_idx (nullable), tau, eta, c: as in
+ *             eqb_route_topk / lei_inject_grad;
+ *   mb_offsets_host host copy of mb_offsets (nullable; validated when given)
+ *   r         global target rank; r <= 0 means eqb_target_rank(T, E, K)
+ *   loads     device int32 [M,E], overwritten (zeroed by the call)
+ *   b_next    device fp32 [E] (out): the bias for the next step
+ *   grad_s    device fp32 [T,E] updated in place, or NULL (no LEI)
+ *   workspace device buffer of at least eqb_layer_workspace_bytes(E) bytes,
+ *             256-byte aligned, owned by the caller; its contents on return
+ *             are the step's histograms and selections
+ * Histograms are local to the call, so this entry point is for a single
+ * process; a multi-GPU caller all-reduces between the per-pass calls. */
+eqb_status eqb_layer_step(const eqb_bf16 *z, const float *b, int64_t T, int32_t E, int32_t K,
+                          const int64_t *mb_offsets, const int64_t *mb_offsets_host, int32_t M,
+                          int64_t r, int32_t *topk_idx, float *tau, int32_t *loads, float *b_next,
+                          float *grad_s, float eta, float c, void *workspace,
+                          size_t workspace_bytes, int32_t *err_flag, void *stream);
 
 /* Router logits, Sec. 2 (Eq. 1: z_t = W_r x_t):
  *   z[t, e] = bf16_rne(sum_k x[t, k] * W_r[e, k]),

@@ -30,7 +30,8 @@ from ._lib import STATUS, EqbError, load
 __all__ = [
     "EqbError", "STATUS", "load", "eqb_target_rank", "eqb_route_topk", "eqb_margin_hist_pass1",
     "eqb_margin_hist_pass2", "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad",
-    "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits",
+    "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
+    "eqb_layer_step",
 ]
 
 
@@ -155,6 +156,45 @@ def eqb_router_logits(x, W_r, z=None, err_flag=None, stream=None):
     _check(load().eqb_router_logits(_p(x), _p(W_r), T, d, E, _p(z), _p(err_flag), _stream(stream)),
            "eqb_router_logits")
     return z
+
+
+def eqb_layer_workspace_bytes(E: int) -> int:
+    return int(load().eqb_layer_workspace_bytes(E))
+
+
+def eqb_layer_step(z, b, K, mb_offsets, loads, b_next, workspace, tau=None, topk_idx=None,
+                   grad_s=None, eta=0.0, c=0.0, mb_offsets_host=None, r=0, err_flag=None,
+                   stream=None):
+    """The whole routing-balance step of one layer in one library call (see
+    eqb.h).  workspace: uint8 CUDA tensor of eqb_layer_workspace_bytes(E)
+    bytes.  mb_offsets_host: optional int64 host copy of the offsets, checked
+    by the library before anything is launched."""
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(b, torch.float32, "b", (E,))
+    _need(mb_offsets, torch.int64, "mb_offsets")
+    M = mb_offsets.numel() - 1
+    _need(loads, torch.int32, "loads", (M, E))
+    _need(b_next, torch.float32, "b_next", (E,))
+    _need(workspace, torch.uint8, "workspace")
+    if tau is None:
+        tau = torch.empty(T, dtype=torch.float32, device=z.device)
+    _need(tau, torch.float32, "tau", (T,))
+    _need(topk_idx, torch.int32, "topk_idx", (T, K))
+    _need(grad_s, torch.float32, "grad_s", (T, E) if grad_s is not None else None)
+    _need(err_flag, torch.int32, "err_flag")
+    host = None
+    if mb_offsets_host is not None:
+        import numpy as np
+        host = np.ascontiguousarray(np.asarray(mb_offsets_host), dtype=np.int64)
+        if host.shape != (M + 1,):
+            raise ValueError("mb_offsets_host must have M+1 entries")
+    hp = None if host is None else host.ctypes.data_as(ctypes.c_void_p)
+    rc = load().eqb_layer_step(_p(z), _p(b), T, E, K, _p(mb_offsets), hp, M, int(r), _p(topk_idx),
+                               _p(tau), _p(loads), _p(b_next), _p(grad_s), float(eta), float(c),
+                               _p(workspace), workspace.numel(), _p(err_flag), _stream(stream))
+    _check(rc, "eqb_layer_step")
+    return tau
 
 
 class EqbWorkspace:

@@ -15,7 +15,8 @@ LIB_PATH = os.path.join(HERE, "libeqb.so")
 EXPORTS = (
     "eqb_status_string", "eqb_version", "eqb_target_rank", "eqb_route_topk",
     "eqb_margin_hist_pass1", "eqb_margin_hist_pass2", "eqb_select_quantile",
-    "eqb_bias_update", "lei_inject_grad", "eqb_router_logits",
+    "eqb_bias_update", "lei_inject_grad", "eqb_router_logits", "eqb_layer_workspace_bytes",
+    "eqb_layer_step",
 )
 
 STATUS = {0: "EQB_OK", 1: "EQB_ERR_INVALID_ARG", 2: "EQB_ERR_UNSUPPORTED", 3: "EQB_ERR_CUDA",
@@ -51,6 +52,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
             "eqb_bias_update": [P, i32, P, P],
             "lei_inject_grad": [P, P, P, i32, i64, i32, i32, f32, f32, P],
             "eqb_router_logits": [P, P, i64, i32, i32, P, P, P],
+            "eqb_layer_step": [P, P, i64, i32, i32, P, P, i32, i64, P, P, P, P, P, f32, f32, P,
+                               ctypes.c_size_t, P, P],
         }
         for name, args in sigs.items():
             fn = getattr(lib, name)
@@ -60,6 +63,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.eqb_status_string.restype = ctypes.c_char_p
         lib.eqb_version.argtypes = []
         lib.eqb_version.restype = ctypes.c_int
+        lib.eqb_layer_workspace_bytes.argtypes = [i32]
+        lib.eqb_layer_workspace_bytes.restype = ctypes.c_size_t
         lib.eqb_target_rank.argtypes = [i64, i32, i32]
         lib.eqb_target_rank.restype = i64
         if path is None:

@@ -6,7 +6,7 @@
 
 #include <atomic>
 
-#include "../../include/eqb.h"
+#include "eqb.h"
 #include "eqb_internal.h"
 
 namespace eqb {
@@ -93,7 +93,7 @@ eqb_status eqb_route_topk(const eqb_bf16* z, const float* b, int64_t T, int32_t 
       !aligned(loads, 4) || !aligned(hist_hi, 4) || !aligned(mb_offsets, 8) || !aligned(err_flag, 4))
     return EQB_ERR_INVALID_ARG;
   if (T == 0) return EQB_OK;
-  eqb::RouteArgs a{z, b, T, E, K, mb_offsets, M, topk_idx, tau, loads, err_flag};
+  eqb::RouteArgs a{z, b, T, E, K, mb_offsets, M, 0, topk_idx, tau, loads, err_flag};
   int rc = eqb::launch_route(a, as_stream(stream));
   if (rc != 0 || !hist_hi) return to_status(rc);
   eqb::HistArgs h{z, tau, T, E, nullptr, hist_hi, err_flag};
@@ -151,7 +151,7 @@ eqb_status lei_inject_grad(float* grad_s, const int32_t* loads, const int64_t* m
   if (!(eta == eta) || !(c == c)) return EQB_ERR_INVALID_ARG;
   if (!aligned(grad_s, 16) || !aligned(loads, 4) || !aligned(mb_offsets, 8)) return EQB_ERR_INVALID_ARG;
   if (T == 0) return EQB_OK;
-  eqb::LeiArgs a{grad_s, loads, mb_offsets, M, T, E, K, eta, c};
+  eqb::LeiArgs a{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
   return to_status(eqb::launch_lei(a, as_stream(stream)));
 }
 

@@ -30,8 +30,9 @@ struct RouteArgs {
   const float* b;
   int64_t T;
   int E, K;
-  const int64_t* off;
+  const int64_t* off;  // microbatch boundaries, absolute token numbers
   int M;
+  int64_t tbase;       // absolute number of token 0 of this call
   int32_t* idx;
   float* tau;
   int32_t* loads;
@@ -51,8 +52,9 @@ struct HistArgs {
 struct LeiArgs {
   float* g;
   const int32_t* loads;
-  const int64_t* off;
+  const int64_t* off;  // microbatch boundaries, absolute token numbers
   int M;
+  int64_t tbase;       // absolute number of token 0 of this call
   int64_t T;
   int E, K;
   float eta, c;

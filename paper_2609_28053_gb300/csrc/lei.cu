@@ -24,6 +24,7 @@ constexpr int kLeiUnroll = 4;
 __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tokens_per_cta) {
   __shared__ __align__(16) float coef[256];
   __shared__ double red[kLeiThreads / 32];
+  __shared__ double scal[2];
   const int E = a.E, E4 = a.E >> 2;
   const int64_t tb = (int64_t)blockIdx.x * tokens_per_cta;
   const int64_t te = min(tb + tokens_per_cta, a.T);
@@ -34,32 +35,42 @@ __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tok
 
   int64_t t = tb;
   while (t < te) {
-    const int l = microbatch_of(a.off, a.M, t);
-    const int64_t lo = __ldg(a.off + l), hi = __ldg(a.off + l + 1);
+    const int l = microbatch_of(a.off, a.M, t + a.tbase);
+    const int64_t lo = __ldg(a.off + l) - a.tbase, hi = __ldg(a.off + l + 1) - a.tbase;
     // Malformed offsets (off[M] < T) must not stall the loop: tokens past
     // the last boundary are treated as the last microbatch's.
     const int64_t seg_end = (hi > t) ? min(te, hi) : te;
 
-    // ---- coefficients of microbatch l
-    __syncthreads();  // previous segment finished reading coef
-    const double n = (double)(hi - lo);
-    const double fbar = (double)a.K * n / (double)E;
+    // ---- coefficients of microbatch l.  fp64 throughput is low on this
+    // part, so each thread does only a multiply-add and a multiply; the
+    // reciprocal of the target load and tanh are formed once per block.
+    __syncthreads();  // previous segment finished reading coef and scal
+    if (threadIdx.x == 0) {
+      const double n = (double)(hi - lo);
+      scal[0] = n > 0.0 ? (double)E / ((double)a.K * n) : 0.0;  // 1 / fbar
+    }
+    __syncthreads();
+    const double inv_fbar = scal[0];
     double rho = 0.0;
-    if (threadIdx.x < E && n > 0.0)
-      rho = (double)__ldg(a.loads + (int64_t)l * E + threadIdx.x) / fbar - 1.0;
+    if (threadIdx.x < E && inv_fbar > 0.0)
+      rho = (double)__ldg(a.loads + (int64_t)l * E + threadIdx.x) * inv_fbar - 1.0;
     double amax = fabs(rho);
 #pragma unroll
     for (int d = 16; d > 0; d >>= 1) amax = fmax(amax, __shfl_xor_sync(kFull, amax, d));
     if (lane == 0) red[wid] = amax;
     __syncthreads();
-    double rmax = red[0];
-    for (int w = 1; w < (int)(blockDim.x >> 5); ++w) rmax = fmax(rmax, red[w]);
-    double sigma = 1.0;
-    if (a.c > 0.0f) {
-      const double xi = rmax / (double)a.c;
-      sigma = (xi == 0.0) ? 1.0 : tanh(xi) / xi;
+    if (threadIdx.x == 0) {
+      double rmax = red[0];
+      for (int w = 1; w < (int)(blockDim.x >> 5); ++w) rmax = fmax(rmax, red[w]);
+      double sigma = 1.0;
+      if (a.c > 0.0f) {
+        const double xi = rmax / (double)a.c;
+        sigma = (xi == 0.0) ? 1.0 : tanh(xi) / xi;
+      }
+      scal[1] = (double)a.eta * sigma;
     }
-    if (threadIdx.x < E) coef[threadIdx.x] = __double2float_rn((double)a.eta * sigma * rho);
+    __syncthreads();
+    if (threadIdx.x < E) coef[threadIdx.x] = __double2float_rn(scal[1] * rho);
     __syncthreads();
 
     // ---- stream grad_s[t .. seg_end) in float4 units
@@ -109,7 +120,7 @@ int launch_lei(const LeiArgs& a, cudaStream_t s) {
   DeviceInfo di;
   if (int rc = device_info(&di)) return rc;
   int64_t grid = (int64_t)di.sm_count * 8;
-  // at least 256 tokens per CTA so the per-microbatch prologue stays cheap
+  // at least 256 tokens per CTA so the per-microbatch prologue stays small
   const int64_t max_grid = (a.T + 255) / 256;
   if (grid > max_grid) grid = max_grid;
   if (grid < 1) grid = 1;

@@ -231,6 +231,7 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
 
     // ---- B: per-chunk masks of U >= threshold, chunks with a hit listed
     int cnt = 0;
+#pragma unroll 2
     for (int c = 0; c < nch; ++c) {
       const uint4 w = lds128(rowp + c * 16);
       const uint4 bu = bup4[c];
@@ -257,23 +258,40 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
     for (int j = 0; j < KP1; ++j) { v[j] = -INFINITY; id[j] = 0; }
     // One candidate per lane per iteration: a lane whose current chunk mask
     // is used up loads its next entry, so the warp runs for the largest
-    // candidate count of its lanes.
+    // candidate count of its lanes.  The next candidate's z and b are read
+    // one iteration ahead, off the insertion's critical path.
     int ei = 0, cbase = 0;
     uint32_t m = 0u;
-    for (;;) {
+    auto next = [&](int& e_out) -> bool {
       if (m == 0u && ei < cnt) {
         const uint32_t en = ent[(ei << 5) | lane];
         cbase = static_cast<int>(en >> 8) * 8;
         m = en & 0xffu;
         ++ei;
       }
-      if (!__any_sync(kFull, m != 0u)) break;
-      if (m != 0u) {
-        const int e = cbase + __ffs(m) - 1;
-        m &= m - 1u;
-        const float s = bf16_bits_to_f32(*reinterpret_cast<const uint16_t*>(rowp + 2 * e)) + bs[e];
-        insert_sorted<KP1>(v, id, s, e);
+      if (m == 0u) return false;
+      e_out = cbase + __ffs(m) - 1;
+      m &= m - 1u;
+      return true;
+    };
+    int e_cur = 0;
+    bool have = next(e_cur);
+    uint32_t zc = have ? *reinterpret_cast<const uint16_t*>(rowp + 2 * e_cur) : 0u;
+    float bc = have ? bs[e_cur] : 0.f;
+    while (__any_sync(kFull, have)) {
+      int e_nxt = 0;
+      const bool have_nxt = next(e_nxt);
+      uint32_t zn = 0u;
+      float bn = 0.f;
+      if (have_nxt) {
+        zn = *reinterpret_cast<const uint16_t*>(rowp + 2 * e_nxt);
+        bn = bs[e_nxt];
       }
+      if (have) insert_sorted<KP1>(v, id, bf16_bits_to_f32(zc) + bc, e_cur);
+      have = have_nxt;
+      e_cur = e_nxt;
+      zc = zn;
+      bc = bn;
     }
     __syncwarp();
 
@@ -292,7 +310,7 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
       }
     }
     if (a.loads) {
-      const int l = valid ? microbatch_of(a.off, a.M, t) : -1;
+      const int l = valid ? microbatch_of(a.off, a.M, t + a.tbase) : -1;
       const int l0 = __shfl_sync(kFull, l, 0);
       if (l0 != cur_mb) {
         flush_loads();

@@ -1,0 +1,99 @@
+// step.cu -- one call for a layer's whole routing-balance step (the host-side
+// order of launches; every step runs in the library's kernels).
+//
+// Order of work, as in the paper: routing (Sec. 2), Algorithm 1's coarse
+// pass, selection, fine pass, selection and the Eq. (2) bias update, then
+// Load-Error Injection (Sec. 4, Eqs. LEI and norm).  All on one stream.
+#include <cuda_runtime.h>
+#include <stdint.h>
+
+#include "eqb.h"
+#include "eqb_internal.h"
+
+namespace {
+
+size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+struct Workspace {
+  int32_t* H;
+  int32_t* L;
+  uint8_t* u;
+  int32_t* rho;
+  uint16_t* q;
+};
+
+// Carve the caller's workspace (or, with base == NULL, only measure it).
+size_t carve(void* base, int E, Workspace* w) {
+  size_t off = 0;
+  auto take = [&](size_t n) {
+    uint8_t* p = base ? static_cast<uint8_t*>(base) + off : nullptr;
+    off = align_up(off + n, 256);
+    return p;
+  };
+  w->H = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 256 * 4));
+  w->L = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 256 * 4));
+  w->u = take(static_cast<size_t>(E));
+  w->rho = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 4));
+  w->q = reinterpret_cast<uint16_t*>(take(static_cast<size_t>(E) * 2));
+  return off;
+}
+
+inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
+inline eqb_status st(int rc) { return static_cast<eqb_status>(rc); }
+
+}  // namespace
+
+extern "C" {
+
+size_t eqb_layer_workspace_bytes(int32_t E) {
+  if (E < 1) return 0;
+  Workspace w;
+  return carve(nullptr, E, &w);
+}
+
+eqb_status eqb_layer_step(const eqb_bf16* z, const float* b, int64_t T, int32_t E, int32_t K,
+                          const int64_t* mb_offsets, const int64_t* mb_offsets_host, int32_t M,
+                          int64_t r, int32_t* topk_idx, float* tau, int32_t* loads, float* b_next,
+                          float* grad_s, float eta, float c, void* workspace, size_t workspace_bytes,
+                          int32_t* err_flag, void* stream) {
+  if (T < 1 || E < 2 || K < 1 || K >= E || M < 1) return EQB_ERR_INVALID_ARG;
+  if (E > 256 || (E % 8) != 0 || K + 1 > 32) return EQB_ERR_UNSUPPORTED;
+  if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
+  if (!z || !b || !mb_offsets || !tau || !loads || !b_next || !workspace) return EQB_ERR_INVALID_ARG;
+  if (grad_s && (!(eta == eta) || !(c == c))) return EQB_ERR_INVALID_ARG;
+  if (!aligned(z, 16) || !aligned(b, 4) || !aligned(mb_offsets, 8) || !aligned(topk_idx, 4) ||
+      !aligned(tau, 4) || !aligned(loads, 4) || !aligned(b_next, 4) || !aligned(grad_s, 16) ||
+      !aligned(workspace, 256) || !aligned(err_flag, 4))
+    return EQB_ERR_INVALID_ARG;
+  Workspace w;
+  if (workspace_bytes < carve(workspace, E, &w)) return EQB_ERR_INVALID_ARG;
+  if (mb_offsets_host) {
+    if (mb_offsets_host[0] != 0 || mb_offsets_host[M] != T) return EQB_ERR_INVALID_ARG;
+    for (int l = 0; l < M; ++l)
+      if (mb_offsets_host[l + 1] < mb_offsets_host[l]) return EQB_ERR_INVALID_ARG;
+  }
+  if (r <= 0) r = eqb_target_rank(T, E, K);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+
+  if (cudaMemsetAsync(w.H, 0, static_cast<size_t>(E) * 256 * 4, s) != cudaSuccess ||
+      cudaMemsetAsync(w.L, 0, static_cast<size_t>(E) * 256 * 4, s) != cudaSuccess ||
+      cudaMemsetAsync(loads, 0, static_cast<size_t>(M) * E * 4, s) != cudaSuccess)
+    return EQB_ERR_CUDA;
+
+  eqb::RouteArgs ra{z, b, T, E, K, mb_offsets, M, 0, topk_idx, tau, loads, err_flag};
+  if (int rc = eqb::launch_route(ra, s)) return st(rc);
+  eqb::HistArgs h1{z, tau, T, E, nullptr, w.H, err_flag};
+  if (int rc = eqb::launch_hist(h1, 1, s)) return st(rc);
+  if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
+  eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};
+  if (int rc = eqb::launch_hist(h2, 2, s)) return st(rc);
+  if (int rc = eqb::launch_select(w.L, E, 2, r, w.u, w.rho, w.q, err_flag, s)) return st(rc);
+  if (int rc = eqb::launch_bias_update(w.q, E, b_next, s)) return st(rc);
+  if (grad_s) {
+    eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
+    if (int rc = eqb::launch_lei(la, s)) return st(rc);
+  }
+  return EQB_OK;
+}
+
+}  // extern "C"

@@ -120,3 +120,32 @@ def test_router_logits_rejects(lib):
     assert f(FAKE, FAKE, -1, 4096, 128, FAKE, NULL, NULL) == INVALID
     assert f(MISALIGNED, FAKE, 10, 4096, 128, FAKE, NULL, NULL) == INVALID
     assert f(FAKE, FAKE, 0, 4096, 128, FAKE, NULL, NULL) == 0
+
+
+def test_layer_step_workspace_size(lib):
+    assert lib.eqb_layer_workspace_bytes(256) >= 2 * 256 * 256 * 4 + 256 * 7
+    assert lib.eqb_layer_workspace_bytes(256) % 256 == 0
+    assert lib.eqb_layer_workspace_bytes(0) == 0
+
+
+def test_layer_step_rejects(lib):
+    import numpy as np
+    f = lib.eqb_layer_step
+    ws = lib.eqb_layer_workspace_bytes(64)
+    good = np.array([0, 40, 100], np.int64)
+    bad = np.array([0, 60, 50], np.int64)
+    short = np.array([0, 40, 99], np.int64)
+    fl = ctypes.c_float(0.0)
+
+    def call(T=100, E=64, K=8, off_h=good, ws_bytes=ws, workspace=FAKE, z=FAKE, M=2):
+        hp = None if off_h is None else off_h.ctypes.data_as(ctypes.c_void_p)
+        return f(z, FAKE, T, E, K, FAKE, hp, M, 0, FAKE, FAKE, FAKE, FAKE, NULL, fl, fl,
+                 workspace, ws_bytes, NULL, NULL)
+    assert call(off_h=bad) == INVALID          # decreasing offsets
+    assert call(off_h=short) == INVALID        # offsets do not end at T
+    assert call(ws_bytes=ws - 1) == INVALID    # workspace too small
+    assert call(workspace=NULL) == INVALID
+    assert call(workspace=ctypes.c_void_p(0x10010)) == INVALID  # not 256-byte aligned
+    assert call(z=NULL) == INVALID
+    assert call(T=0) == INVALID
+    assert call(E=60) == UNSUPPORTED

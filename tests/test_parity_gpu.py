@@ -346,3 +346,41 @@ def test_bias_update_exact_against_oracle(kind):
     eqb.eqb_bias_update(torch.from_numpy(q.view(np.int16)).view(torch.bfloat16).cuda(), bd)
     torch.cuda.synchronize()
     assert np.array_equal(bits_f32(bd.cpu().numpy()), bits_f32(want))
+
+
+# ------------------------------------------------------------- one-call step
+
+@pytest.mark.parametrize("T,E,K,M", [(300000, 256, 8, 11), (140000, 128, 6, 4), (5000, 64, 8, 3)])
+def test_layer_step_matches_oracle(T, E, K, M):
+    """eqb_layer_step reproduces the oracle: routing, loads and the bias
+    update bit for bit, LEI within tolerance."""
+    z, b = rand_case(T, E, seed=T + E + K)
+    off = ragged_offsets(T, M, seed=M)
+    off[1] = off[2]  # one empty microbatch
+    g = (np.random.default_rng(T).standard_normal((T, E)) * 0.1).astype(np.float32)
+    eta, c = 0.25, 1.0
+    o = oracle_forward(z, b, K, off)
+    g_ref, _ = oracle.lei(g, o["loads"], off, K, eta, c)
+
+    zd, bd = to_dev_bf16(z), torch.from_numpy(b).cuda()
+    offd = torch.from_numpy(off).cuda()
+    idx = Guarded((T, K), torch.int32)
+    tau = Guarded((T,), torch.float32)
+    loads = Guarded((M, E), torch.int32, fill=99)
+    bn = Guarded((E,), torch.float32)
+    G = Guarded((T, E), torch.float32)
+    G.view.copy_(torch.from_numpy(g))
+    ws = torch.zeros(eqb.eqb_layer_workspace_bytes(E), dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    eqb.eqb_layer_step(zd, bd, K, offd, loads.view, bn.view, ws, tau=tau.view, topk_idx=idx.view,
+                       grad_s=G.view, eta=eta, c=c, mb_offsets_host=off, err_flag=err)
+    torch.cuda.synchronize()
+    for buf in (idx, tau, loads, bn, G):
+        assert buf.intact()
+    assert err.item() == 0
+    assert np.array_equal(idx.view.cpu().numpy(), o["idx"])
+    assert np.array_equal(bits_f32(tau.view.cpu().numpy()), bits_f32(o["tau"]))
+    assert np.array_equal(loads.view.cpu().numpy(), o["loads"])
+    assert np.array_equal(bits_f32(bn.view.cpu().numpy()), bits_f32(o["b_next"]))
+    got = G.view.cpu().numpy().astype(np.float64)
+    assert np.all(np.abs(got - g_ref) <= LEI_ATOL + LEI_RTOL * np.abs(g_ref))
