@@ -181,6 +181,29 @@ eqb_status eqb_layer_step(const eqb_bf16 *z, const float *b, int64_t T, int32_t 
                           float *grad_s, float eta, float c, void *workspace,
                           size_t workspace_bytes, int32_t *err_flag, void *stream);
 
+/* eqb_layer_step for callers that cannot allocate device memory (no
+ * counterpart in the paper; a library convenience).  Plugins hosted by a
+ * framework or server that owns all device memory through its own pool, and
+ * code that must not stall on or fail at an allocation, can call this
+ * instead: it takes the same inputs and outputs but no workspace, and uses a
+ * scratch array compiled into the library.
+ *   - The scratch holds the step's histograms and selections for E <= 256
+ *     (526,080 bytes); E > 256 returns EQB_ERR_UNSUPPORTED.  Every GPU that
+ *     loads the library keeps this array until the process exits.
+ *   - The first call on each device looks up the array's device address
+ *     (cudaGetSymbolAddress) with that device current; make it before any
+ *     stream capture.  It allocates nothing.
+ *   - All calls on a device share the array, which keeps the previous
+ *     call's contents (the step zeroes the histograms before counting);
+ *     calls that overlap on the GPU race on it.
+ * Arguments and results are those of eqb_layer_step. */
+eqb_status eqb_layer_step_noalloc(const eqb_bf16 *z, const float *b, int64_t T, int32_t E,
+                                  int32_t K, const int64_t *mb_offsets,
+                                  const int64_t *mb_offsets_host, int32_t M, int64_t r,
+                                  int32_t *topk_idx, float *tau, int32_t *loads, float *b_next,
+                                  float *grad_s, float eta, float c, int32_t *err_flag,
+                                  void *stream);
+
 /* Router logits, Sec. 2 (Eq. 1: z_t = W_r x_t):
  *   z[t, e] = bf16_rne(sum_k x[t, k] * W_r[e, k]),
  * bf16 inputs, fp32 accumulation on the tensor cores (tcgen05, accumulators

@@ -31,7 +31,7 @@ __all__ = [
     "EqbError", "STATUS", "load", "eqb_target_rank", "eqb_route_topk", "eqb_margin_hist_pass1",
     "eqb_margin_hist_pass2", "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad",
     "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
-    "eqb_layer_step",
+    "eqb_layer_step", "eqb_layer_step_noalloc",
 ]
 
 
@@ -194,6 +194,40 @@ def eqb_layer_step(z, b, K, mb_offsets, loads, b_next, workspace, tau=None, topk
                                _p(tau), _p(loads), _p(b_next), _p(grad_s), float(eta), float(c),
                                _p(workspace), workspace.numel(), _p(err_flag), _stream(stream))
     _check(rc, "eqb_layer_step")
+    return tau
+
+
+def eqb_layer_step_noalloc(z, b, K, mb_offsets, loads, b_next, tau=None, topk_idx=None,
+                           grad_s=None, eta=0.0, c=0.0, mb_offsets_host=None, r=0, err_flag=None,
+                           stream=None):
+    """eqb_layer_step without a workspace argument, for callers that cannot
+    allocate device memory: the step's scratch is an array inside the
+    library (E <= 256).  Calls that overlap on the GPU share that array and
+    race; the first call on a device should come before any stream capture."""
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(b, torch.float32, "b", (E,))
+    _need(mb_offsets, torch.int64, "mb_offsets")
+    M = mb_offsets.numel() - 1
+    _need(loads, torch.int32, "loads", (M, E))
+    _need(b_next, torch.float32, "b_next", (E,))
+    if tau is None:
+        tau = torch.empty(T, dtype=torch.float32, device=z.device)
+    _need(tau, torch.float32, "tau", (T,))
+    _need(topk_idx, torch.int32, "topk_idx", (T, K))
+    _need(grad_s, torch.float32, "grad_s", (T, E) if grad_s is not None else None)
+    _need(err_flag, torch.int32, "err_flag")
+    hp = None
+    if mb_offsets_host is not None:
+        import numpy as np
+        host = np.ascontiguousarray(np.asarray(mb_offsets_host), dtype=np.int64)
+        if host.shape != (M + 1,):
+            raise ValueError("mb_offsets_host must have M+1 entries")
+        hp = host.ctypes.data_as(ctypes.c_void_p)
+    rc = load().eqb_layer_step_noalloc(_p(z), _p(b), T, E, K, _p(mb_offsets), hp, M, int(r),
+                                       _p(topk_idx), _p(tau), _p(loads), _p(b_next), _p(grad_s),
+                                       float(eta), float(c), _p(err_flag), _stream(stream))
+    _check(rc, "eqb_layer_step_noalloc")
     return tau
 
 
