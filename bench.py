@@ -112,8 +112,9 @@ class Step:
 
     workload 'global': logits resident in HBM (T=2,097,152, E=256, K=8).
     workload 'router': the router projection on the tensor cores first
-    (x [T,4096] bf16, W_r [128,4096]), then the same path on its logits; the
-    bias produced by a step is the next step's bias (Eq. 2)."""
+    (x [T,4096] bf16, W_r [128,4096]), each token routed from the
+    projection's accumulators in the same kernel, then the same path on its
+    logits; the bias produced by a step is the next step's bias (Eq. 2)."""
 
     def __init__(self, workload, T, dev, seed_shift=0):
         import paper_2609_28053_gb300 as eqb
@@ -142,8 +143,8 @@ class Step:
         self.r_global = None
         self.off_h = even_offsets(T, self.M)
         self.workspace = torch.zeros(eqb.eqb_layer_workspace_bytes(E), dtype=torch.uint8, device=dev)
-        self.names = (["router_logits"] if workload == "router" else []) + [
-            "route_topk", "margin_hist_pass1", "select_pass1", "margin_hist_pass2",
+        self.names = (["router_route"] if workload == "router" else ["route_topk"]) + [
+            "margin_hist_pass1", "select_pass1", "margin_hist_pass2",
             "select_pass2", "bias_update", "lei_inject_grad"]
 
     def run_step(self, stream):
@@ -151,13 +152,16 @@ class Step:
         both histogram passes, selections, the bias update and LEI."""
         eqb = self.eqb
         if self.workload == "router":
-            eqb.eqb_router_logits(self.x, self.W, self.z, self.ws.err, stream)
+            eqb.eqb_router_layer_step(self.x, self.W, self.b, self.K, self.off, self.loads, self.b_next,
+                                      self.workspace, z=self.z, tau=self.tau, topk_idx=self.idx,
+                                      grad_s=self.g, eta=ETA, c=C_NORM, mb_offsets_host=self.off_h,
+                                      r=self.r_global or 0, err_flag=self.ws.err, stream=stream)
+            self.b.copy_(self.b_next)  # b^(q+1) routes step q+1
+            return
         eqb.eqb_layer_step(self.z, self.b, self.K, self.off, self.loads, self.b_next, self.workspace,
                            tau=self.tau, topk_idx=self.idx, grad_s=self.g, eta=ETA, c=C_NORM,
                            mb_offsets_host=self.off_h, r=self.r_global or 0, err_flag=self.ws.err,
                            stream=stream)
-        if self.workload == "router":
-            self.b.copy_(self.b_next)  # b^(q+1) routes step q+1
 
     def run(self, stream, world=1, events=None, z=None, g=None):
         """Enqueue one step.  `events` (optional) is a list of (start, end)
@@ -166,7 +170,6 @@ class Step:
         z = self.z if z is None else z
         g = self.g if g is None else g
         r = self.r_global or eqb.eqb_target_rank(self.T * world, self.E, self.K)
-        i0 = 0
 
         def rec(i, fn):
             if events is not None:
@@ -180,29 +183,31 @@ class Step:
         ws.err.zero_()
         self.loads.zero_()
         if self.workload == "router":
-            rec(0, lambda: eqb.eqb_router_logits(self.x, self.W, z, ws.err, stream))
-            i0 = 1
-        rec(i0 + 0, lambda: eqb.eqb_route_topk(z, self.b, self.K, self.off, self.idx, self.tau,
-                                               self.loads, None, ws.err, stream))
-        rec(i0 + 1, lambda: eqb.eqb_margin_hist_pass1(z, self.tau, ws.hist_hi, ws.err, stream))
+            rec(0, lambda: eqb.eqb_router_route(self.x, self.W, self.b, self.K, self.off, z, self.idx,
+                                                self.tau, self.loads, ws.err, stream))
+        else:
+            rec(0, lambda: eqb.eqb_route_topk(z, self.b, self.K, self.off, self.idx, self.tau,
+                                              self.loads, None, ws.err, stream))
+        rec(1, lambda: eqb.eqb_margin_hist_pass1(z, self.tau, ws.hist_hi, ws.err, stream))
         if world > 1:
             torch.distributed.all_reduce(ws.hist_hi)
-        rec(i0 + 2, lambda: eqb.eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream))
-        rec(i0 + 3, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
+        rec(2, lambda: eqb.eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream))
+        rec(3, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
         if world > 1:
             torch.distributed.all_reduce(ws.hist_lo)
-        rec(i0 + 4, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err,
+        rec(4, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err,
                                                     stream))
-        rec(i0 + 5, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
-        rec(i0 + 6, lambda: eqb.lei_inject_grad(g, self.loads, self.off, self.K, ETA, C_NORM, stream))
+        rec(5, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
+        rec(6, lambda: eqb.lei_inject_grad(g, self.loads, self.off, self.K, ETA, C_NORM, stream))
         if self.workload == "router":
             self.b.copy_(self.b_next)  # b^(q+1) routes step q+1
 
     def launches_per_step(self):
         """Kernels of this library launched by one timed step (memsets and
         torch copies excluded): routing, two histogram passes, two
-        selections, the bias update and LEI (+ the router GEMM)."""
-        return 7 + (1 if self.workload == "router" else 0)
+        selections, the bias update and LEI (for the router workload the
+        routing kernel is the router projection with routing)."""
+        return 7
 
     def algorithmic_bytes(self):
         """Bytes the two-pass method must move per step (see the design notes):
@@ -216,8 +221,10 @@ class Step:
              "lei_inject_grad": 8 * T * E,
              "path": 12 * T * E + 8 * T + 4 * T * K}
         if self.workload == "router":
-            d["router_logits"] = 2 * T * self.d + 2 * E * self.d + 2 * T * E
-            d["path"] += d["router_logits"]
+            # the projection reads x and W_r and writes z; routing from its
+            # accumulators then adds only idx and tau
+            d["router_route"] = 2 * T * self.d + 2 * E * self.d + 2 * T * E + 4 * T * K + 4 * T
+            d["path"] += d["router_route"] - d.pop("route_topk")
         return d
 
 

@@ -221,6 +221,45 @@ eqb_status eqb_layer_step_noalloc(const eqb_bf16 *z, const float *b, int64_t T, 
 eqb_status eqb_router_logits(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t T, int32_t d,
                              int32_t E, eqb_bf16 *z, int32_t *err_flag, void *stream);
 
+/* Router logits and routing in one kernel: eqb_router_logits followed by
+ * eqb_route_topk (without hist_hi), with each token routed straight from the
+ * tensor-memory accumulator of its row, so z is written once and not read
+ * back.  The paper computes the same two steps one after the other (Sec. 2,
+ * Eq. 1, then top-K of s = z + b); fusing them is a property of this library.
+ *   x, W_r, z   as in eqb_router_logits; z is still written (the EQB passes
+ *               and LEI read it)
+ *   b, K, mb_offsets, M, topk_idx, tau, loads, err_flag
+ *               as in eqb_route_topk: topk_idx [T,K] (nullable), tau [T],
+ *               loads [M,E] += (nullable; then mb_offsets may be NULL)
+ * Results equal those of the two calls made one after the other on the same
+ * inputs, bit for bit.  err_flag: EQB_ERR_NONFINITE as in eqb_route_topk,
+ * EQB_ERR_CUDA as in eqb_router_logits.
+ * Supported: E in {64, 128}, 1 <= K <= 8, K < E, d a positive multiple of
+ * 64, 0 <= T <= 2^31 - 2^24; other shapes return EQB_ERR_UNSUPPORTED (make
+ * the two calls instead). */
+eqb_status eqb_router_route(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t T, int32_t d,
+                            int32_t E, int32_t K, const float *b, const int64_t *mb_offsets,
+                            int32_t M, eqb_bf16 *z, int32_t *topk_idx, float *tau,
+                            int32_t *loads, int32_t *err_flag, void *stream);
+
+/* The routing-balance step of one layer from the router input: the router
+ * projection z = bf16(x W_r^T) (Sec. 2, Eq. 1) followed by everything
+ * eqb_layer_step does.  For E in {64, 128} and K <= 8 the projection and the
+ * routing run as one kernel (eqb_router_route); otherwise as
+ * eqb_router_logits then eqb_route_topk.  The other steps are those of
+ * eqb_layer_step, and so are the arguments from b on; z is an output here
+ * (device bf16 [T,E], 16-byte aligned).
+ *   x, W_r, d   as in eqb_router_logits.
+ * Returns EQB_ERR_UNSUPPORTED for d not a multiple of 64 or E not a
+ * multiple of 16, beside eqb_layer_step's own conditions. */
+eqb_status eqb_router_layer_step(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t T, int32_t d,
+                                 int32_t E, int32_t K, const float *b,
+                                 const int64_t *mb_offsets, const int64_t *mb_offsets_host,
+                                 int32_t M, int64_t r, eqb_bf16 *z, int32_t *topk_idx,
+                                 float *tau, int32_t *loads, float *b_next, float *grad_s,
+                                 float eta, float c, void *workspace, size_t workspace_bytes,
+                                 int32_t *err_flag, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

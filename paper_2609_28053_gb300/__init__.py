@@ -31,7 +31,7 @@ __all__ = [
     "EqbError", "STATUS", "load", "eqb_target_rank", "eqb_route_topk", "eqb_margin_hist_pass1",
     "eqb_margin_hist_pass2", "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad",
     "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
-    "eqb_layer_step", "eqb_layer_step_noalloc",
+    "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route", "eqb_router_layer_step",
 ]
 
 
@@ -158,6 +158,35 @@ def eqb_router_logits(x, W_r, z=None, err_flag=None, stream=None):
     return z
 
 
+def eqb_router_route(x, W_r, b, K, mb_offsets=None, z=None, topk_idx=None, tau=None, loads=None,
+                     err_flag=None, stream=None):
+    """Router logits and routing in one kernel (see eqb.h): z = bf16(x W_r^T)
+    and, from the same accumulators, eqb_route_topk's topk_idx, tau and loads
+    (accumulated into).  E in {64, 128}, K <= 8.  Returns (z, topk_idx, tau)."""
+    T, d = x.shape
+    E = W_r.shape[0]
+    _need(x, torch.bfloat16, "x")
+    _need(W_r, torch.bfloat16, "W_r", (E, d))
+    _need(b, torch.float32, "b", (E,))
+    if z is None:
+        z = torch.empty((T, E), dtype=torch.bfloat16, device=x.device)
+    if tau is None:
+        tau = torch.empty(T, dtype=torch.float32, device=x.device)
+    _need(z, torch.bfloat16, "z", (T, E))
+    _need(tau, torch.float32, "tau", (T,))
+    _need(topk_idx, torch.int32, "topk_idx", (T, K))
+    M = 0
+    if mb_offsets is not None:
+        _need(mb_offsets, torch.int64, "mb_offsets")
+        M = mb_offsets.numel() - 1
+    _need(loads, torch.int32, "loads", (M, E) if loads is not None else None)
+    _need(err_flag, torch.int32, "err_flag")
+    _check(load().eqb_router_route(_p(x), _p(W_r), T, d, E, K, _p(b), _p(mb_offsets), M, _p(z),
+                                   _p(topk_idx), _p(tau), _p(loads), _p(err_flag), _stream(stream)),
+           "eqb_router_route")
+    return z, topk_idx, tau
+
+
 def eqb_layer_workspace_bytes(E: int) -> int:
     return int(load().eqb_layer_workspace_bytes(E))
 
@@ -195,6 +224,47 @@ def eqb_layer_step(z, b, K, mb_offsets, loads, b_next, workspace, tau=None, topk
                                _p(workspace), workspace.numel(), _p(err_flag), _stream(stream))
     _check(rc, "eqb_layer_step")
     return tau
+
+
+def eqb_router_layer_step(x, W_r, b, K, mb_offsets, loads, b_next, workspace, z=None, tau=None,
+                          topk_idx=None, grad_s=None, eta=0.0, c=0.0, mb_offsets_host=None, r=0,
+                          err_flag=None, stream=None):
+    """The routing-balance step of one layer from the router input x (see
+    eqb.h): the projection z = bf16(x W_r^T), routed from its accumulators
+    where the shape allows, then everything eqb_layer_step does.  Returns
+    (z, tau)."""
+    T, d = x.shape
+    E = W_r.shape[0]
+    _need(x, torch.bfloat16, "x")
+    _need(W_r, torch.bfloat16, "W_r", (E, d))
+    _need(b, torch.float32, "b", (E,))
+    _need(mb_offsets, torch.int64, "mb_offsets")
+    M = mb_offsets.numel() - 1
+    _need(loads, torch.int32, "loads", (M, E))
+    _need(b_next, torch.float32, "b_next", (E,))
+    _need(workspace, torch.uint8, "workspace")
+    if z is None:
+        z = torch.empty((T, E), dtype=torch.bfloat16, device=x.device)
+    if tau is None:
+        tau = torch.empty(T, dtype=torch.float32, device=x.device)
+    _need(z, torch.bfloat16, "z", (T, E))
+    _need(tau, torch.float32, "tau", (T,))
+    _need(topk_idx, torch.int32, "topk_idx", (T, K))
+    _need(grad_s, torch.float32, "grad_s", (T, E) if grad_s is not None else None)
+    _need(err_flag, torch.int32, "err_flag")
+    host = None
+    if mb_offsets_host is not None:
+        import numpy as np
+        host = np.ascontiguousarray(np.asarray(mb_offsets_host), dtype=np.int64)
+        if host.shape != (M + 1,):
+            raise ValueError("mb_offsets_host must have M+1 entries")
+    hp = None if host is None else host.ctypes.data_as(ctypes.c_void_p)
+    rc = load().eqb_router_layer_step(_p(x), _p(W_r), T, d, E, K, _p(b), _p(mb_offsets), hp, M, int(r),
+                                      _p(z), _p(topk_idx), _p(tau), _p(loads), _p(b_next), _p(grad_s),
+                                      float(eta), float(c), _p(workspace), workspace.numel(),
+                                      _p(err_flag), _stream(stream))
+    _check(rc, "eqb_router_layer_step")
+    return z, tau
 
 
 def eqb_layer_step_noalloc(z, b, K, mb_offsets, loads, b_next, tau=None, topk_idx=None,

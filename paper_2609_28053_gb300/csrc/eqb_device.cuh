@@ -140,4 +140,24 @@ __device__ __forceinline__ void red_shared_add(uint32_t saddr, uint32_t v) {
   asm volatile("red.shared.add.u32 [%0], %1;" ::"r"(saddr), "r"(v));
 }
 
+
+// Insert (s, e) into the descending list (v, id).  Candidates arrive in
+// ascending e, so the new element goes after equal scores: its slot is
+// p = #{j : v[j] >= s}; slots below p keep their entry, slot p takes the new
+// one, slots above p take their predecessor's.  Every slot is computed from
+// the old list, so there is no serial dependency between slots.
+template <int KP1>
+__device__ __forceinline__ void insert_sorted(float (&v)[KP1], int (&id)[KP1], float s, int e) {
+  bool ge[KP1];
+#pragma unroll
+  for (int j = 0; j < KP1; ++j) ge[j] = v[j] >= s;
+#pragma unroll
+  for (int j = KP1 - 1; j >= 1; --j) {
+    v[j] = ge[j] ? v[j] : (ge[j - 1] ? s : v[j - 1]);
+    id[j] = ge[j] ? id[j] : (ge[j - 1] ? e : id[j - 1]);
+  }
+  v[0] = ge[0] ? v[0] : s;
+  id[0] = ge[0] ? id[0] : e;
+}
+
 }  // namespace eqb

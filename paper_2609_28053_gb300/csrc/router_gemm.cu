@@ -134,9 +134,127 @@ __device__ __forceinline__ void tmem_ld32(uint32_t taddr, uint32_t (&r)[32]) {
 
 constexpr uint32_t kTmemCols = 512;  // the whole TMEM of the SM: one CTA per SM
 
+struct GemmArgs {
+  uint16_t* z;
+  int T, d, N, S;
+  int32_t* err;
+  // routing from the accumulator (EC > 0): as in eqb_route_topk
+  const float* b;
+  int K;
+  const int64_t* off;
+  int M;
+  int32_t* idx;
+  float* tau;
+  int32_t* loads;
+};
+
+// Routing state of one token: the running top-(K+1) of s = fp32(z) + b.
+template <int KP1>
+struct TopState {
+  float v[KP1];
+  int id[KP1];
+  bool nan;
+};
+
+// Insert the 32 experts c0 .. c0+31 of one token, given as 16 packed bf16
+// words (the rounded logits), in index order: exact stable insertion, so
+// ties keep the lower index first.
+template <int KP1>
+__device__ __forceinline__ void route_chunk(TopState<KP1>& st, const uint32_t (&p)[16], int c0,
+                                            const float* bsm) {
+#pragma unroll
+  for (int i = 0; i < 32; ++i) {
+    const float zf = (i & 1) ? bf16_hi(p[i >> 1]) : bf16_lo(p[i >> 1]);
+    const float sc = zf + bsm[c0 + i];
+    st.nan |= (sc != sc);
+    insert_sorted<KP1>(st.v, st.id, sc, c0 + i);
+  }
+}
+
+// tau, the top-K list and the loads of one routed token.
+template <int EC, int KP1>
+__device__ __forceinline__ void route_outputs(const TopState<KP1>& st, int row, const GemmArgs& a) {
+  const int K = a.K;
+  float tau_t = st.v[0];
+#pragma unroll
+  for (int j = 1; j < KP1; ++j) tau_t = (j == K) ? st.v[j] : tau_t;
+  a.tau[row] = tau_t;
+  if (st.nan || !isfinite(tau_t)) raise_flag(a.err, kErrNonfinite);
+  if (a.idx) {
+#pragma unroll
+    for (int j = 0; j < KP1; ++j)
+      if (j < K) a.idx[static_cast<int64_t>(row) * K + j] = st.id[j];
+  }
+}
+
+// Per-warp expert counts of the microbatch `cur` not yet added to loads: EC
+// 16-bit counters packed in pairs (expert e in the half e & 1 of word e / 2).
+// A warp adds at most 32 to a counter per tile and flushes before 2047 tiles
+// have passed, so no half overflows.
+template <int EC>
+struct WarpLoads {
+  uint32_t* cnt;  // EC / 2 shared words of this warp
+  int cur;        // microbatch being counted, -1 before the first
+  int tiles;      // tiles counted since the last flush
+};
+
+template <int EC>
+__device__ __forceinline__ void flush_loads(WarpLoads<EC>& wl, const GemmArgs& a, int lane) {
+  __syncwarp();  // every lane's shared-memory adds are visible
+  if (wl.cur >= 0) {
+#pragma unroll
+    for (int w = lane; w < EC / 2; w += 32) {
+      const uint32_t c = wl.cnt[w];
+      if (c) {
+        wl.cnt[w] = 0;
+        int32_t* dst = a.loads + static_cast<int64_t>(wl.cur) * EC + 2 * w;
+        if (c & 0xffffu) atomicAdd(dst, static_cast<int>(c & 0xffffu));
+        if (c >> 16) atomicAdd(dst + 1, static_cast<int>(c >> 16));
+      }
+    }
+  }
+  __syncwarp();
+  wl.tiles = 0;
+}
+
+// Count the top-K experts of this lane's token (if valid) into its
+// microbatch.  Tokens of the microbatch the warp is counting go to shared
+// memory; a tile that starts another microbatch flushes first, and the few
+// tokens of a tile that straddles a boundary go straight to global memory.
+// Called by all 32 lanes.
+template <int EC, int KP1>
+__device__ __forceinline__ void count_loads(WarpLoads<EC>& wl, const TopState<KP1>& st, bool valid, int row,
+                                            const GemmArgs& a, int lane) {
+  const int l = valid ? microbatch_of(a.off, a.M, row) : -1;
+  const bool same = !valid || l == wl.cur;
+  if (!__all_sync(0xffffffffu, same) || wl.tiles >= 2047) {
+    flush_loads<EC>(wl, a, lane);
+    const uint32_t vm = __ballot_sync(0xffffffffu, valid);
+    if (vm) wl.cur = __shfl_sync(0xffffffffu, l, __ffs(vm) - 1);
+  }
+  ++wl.tiles;
+  if (!valid) return;
+  const int K = a.K;
+  if (l == wl.cur) {
+#pragma unroll
+    for (int j = 0; j < KP1; ++j)
+      if (j < K) red_shared_add(smem_u32(wl.cnt + (st.id[j] >> 1)), 1u << ((st.id[j] & 1) * 16));
+  } else {
+#pragma unroll
+    for (int j = 0; j < KP1; ++j)
+      if (j < K) atomicAdd(a.loads + static_cast<int64_t>(l) * EC + st.id[j], 1);
+  }
+}
+
+// EC = 0: the plain GEMM for any supported N.  EC > 0: N = EC and the
+// epilogue also routes each token (K + 1 <= KP1).
+template <int EC, int KP1>
 __global__ void __launch_bounds__(192, 1)
     router_gemm_kernel(const __grid_constant__ CUtensorMap tmx, const __grid_constant__ CUtensorMap tmw,
-                       uint16_t* __restrict__ z, int T, int d, int N, int S, int32_t* err) {
+                       GemmArgs a) {
+  uint16_t* __restrict__ z = a.z;
+  const int T = a.T, d = a.d, N = a.N, S = a.S;
+  int32_t* err = a.err;
   extern __shared__ uint8_t smem_raw[];
   const uint32_t raw = smem_u32(smem_raw);
   const uint32_t base = (raw + 1023u) & ~1023u;  // 1 KiB alignment for the swizzle atoms
@@ -153,8 +271,19 @@ __global__ void __launch_bounds__(192, 1)
   uint32_t* tmem_holder = reinterpret_cast<uint32_t*>(sm + static_cast<size_t>(S) * stage_bytes +
                                                       8u * (2 * S + 5));
   volatile int* abort_flag = reinterpret_cast<volatile int*>(tmem_holder + 1);
+  // routing only: b (EC floats), then 4 warps x EC/2 packed load counters
+  float* bsm = reinterpret_cast<float*>(tmem_holder + 4);
+  uint32_t* lcnt = reinterpret_cast<uint32_t*>(bsm + EC);
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  if (EC > 0) {
+    for (int e = threadIdx.x; e < EC; e += blockDim.x) {
+      const float bv = a.b[e];
+      bsm[e] = bv;
+      if (!isfinite(bv)) raise_flag(err, kErrNonfinite);
+    }
+    for (int w = threadIdx.x; w < 2 * EC; w += blockDim.x) lcnt[w] = 0;
+  }
   const int ntiles = (T + kBM - 1) / kBM;
   const int KB = d / kBK;
 
@@ -237,32 +366,65 @@ __global__ void __launch_bounds__(192, 1)
   } else {
     const int q = warp & 3;  // TMEM lane quarter accessible to this warp
     const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
+    WarpLoads<EC> wl{lcnt + (warp - 2) * (EC / 2), -1, 0};
     int it = 0;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
       const int buf = it & 1;
       const uint32_t use = static_cast<uint32_t>(it >> 1);
-      if (!mbar_wait(accf(buf), use & 1u, abort_flag)) break;
+      // the warp leaves together (the loop body has warp-wide operations)
+      if (!__all_sync(0xffffffffu, mbar_wait(accf(buf), use & 1u, abort_flag))) break;
       tc_fence_after();
       const int row = tile * kBM + q * 32 + lane;
-      for (int c = 0; c < N; c += 32) {
-        uint32_t r[32];
-        tmem_ld32(tmem + lane_base + static_cast<uint32_t>(buf * N + c), r);
-        if (row < T) {
-          uint4* dst = reinterpret_cast<uint4*>(z + static_cast<size_t>(row) * N + c);
+      if constexpr (EC == 0) {
+        for (int c = 0; c < N; c += 32) {
+          uint32_t r[32];
+          tmem_ld32(tmem + lane_base + static_cast<uint32_t>(buf * N + c), r);
+          if (row < T) {
+            uint4* dst = reinterpret_cast<uint4*>(z + static_cast<size_t>(row) * N + c);
 #pragma unroll
-          for (int v = 0; v < 4; ++v) {
-            if (c + 8 * v >= N) break;  // N is a multiple of 16, not always of 32
-            uint4 o;
-            o.x = pack_bf16x2_rn(__uint_as_float(r[8 * v + 0]), __uint_as_float(r[8 * v + 1]));
-            o.y = pack_bf16x2_rn(__uint_as_float(r[8 * v + 2]), __uint_as_float(r[8 * v + 3]));
-            o.z = pack_bf16x2_rn(__uint_as_float(r[8 * v + 4]), __uint_as_float(r[8 * v + 5]));
-            o.w = pack_bf16x2_rn(__uint_as_float(r[8 * v + 6]), __uint_as_float(r[8 * v + 7]));
-            dst[v] = o;
+            for (int v = 0; v < 4; ++v) {
+              if (c + 8 * v >= N) break;  // N is a multiple of 16, not always of 32
+              uint4 o;
+              o.x = pack_bf16x2_rn(__uint_as_float(r[8 * v + 0]), __uint_as_float(r[8 * v + 1]));
+              o.y = pack_bf16x2_rn(__uint_as_float(r[8 * v + 2]), __uint_as_float(r[8 * v + 3]));
+              o.z = pack_bf16x2_rn(__uint_as_float(r[8 * v + 4]), __uint_as_float(r[8 * v + 5]));
+              o.w = pack_bf16x2_rn(__uint_as_float(r[8 * v + 6]), __uint_as_float(r[8 * v + 7]));
+              dst[v] = o;
+            }
           }
         }
+        tc_fence_before();
+        mbar_arrive(acce(buf));
+      } else {
+        // 32 columns at a time: round to bf16, store z, insert into the
+        // token's running top-(K+1).  The accumulator stays in TMEM until the
+        // whole row is read; routing a tile takes far less time than the MMAs
+        // of the next one, which use the other accumulator meanwhile.
+        TopState<KP1> st;
+#pragma unroll
+        for (int j = 0; j < KP1; ++j) { st.v[j] = -INFINITY; st.id[j] = 0; }
+        st.nan = false;
+#pragma unroll 1
+        for (int c = 0; c < EC; c += 32) {
+          uint32_t r[32], p[16];
+          tmem_ld32(tmem + lane_base + static_cast<uint32_t>(buf * EC + c), r);
+#pragma unroll
+          for (int i = 0; i < 16; ++i) p[i] = pack_bf16x2_rn(__uint_as_float(r[2 * i]), __uint_as_float(r[2 * i + 1]));
+          if (row < T) {
+            uint4* dst = reinterpret_cast<uint4*>(z + static_cast<size_t>(row) * EC + c);
+#pragma unroll
+            for (int v = 0; v < 4; ++v) dst[v] = make_uint4(p[4 * v], p[4 * v + 1], p[4 * v + 2], p[4 * v + 3]);
+          }
+          route_chunk<KP1>(st, p, c, bsm);
+        }
+        tc_fence_before();
+        mbar_arrive(acce(buf));
+        if (row < T) route_outputs<EC, KP1>(st, row, a);
+        if (a.loads) count_loads<EC, KP1>(wl, st, row < T, row, a, lane);
       }
-      tc_fence_before();
-      mbar_arrive(acce(buf));
+    }
+    if constexpr (EC > 0) {
+      if (a.loads) flush_loads<EC>(wl, a, lane);
     }
   }
   tc_fence_before();
@@ -309,27 +471,49 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uin
 
 }  // namespace
 
-int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, uint16_t* z,
-                       int32_t* err, cudaStream_t s) {
+namespace {
+
+template <int EC, int KP1>
+int launch_gemm(const uint16_t* x, const uint16_t* W, GemmArgs a, cudaStream_t s) {
   DeviceInfo di;
   if (int rc = device_info(&di)) return rc;
   CUtensorMap tmx, tmw;
-  if (!make_map(&tmx, x, static_cast<uint64_t>(T), static_cast<uint64_t>(d), kBM)) return kErrCuda;
-  if (!make_map(&tmw, W, static_cast<uint64_t>(E), static_cast<uint64_t>(d), static_cast<uint32_t>(E)))
+  if (!make_map(&tmx, x, static_cast<uint64_t>(a.T), static_cast<uint64_t>(a.d), kBM)) return kErrCuda;
+  if (!make_map(&tmw, W, static_cast<uint64_t>(a.N), static_cast<uint64_t>(a.d), static_cast<uint32_t>(a.N)))
     return kErrCuda;
-  const int stage_bytes = (kBM + E) * kBK * 2;
-  const int extra = 1024 + 8 * (2 * 8 + 5) + 16;
+  const int stage_bytes = (kBM + a.N) * kBK * 2;
+  // alignment slack, 2S+5 mbarriers (S <= 8), TMEM address + abort flag, b,
+  // the epilogue warps' load counters
+  const int extra = 1024 + 8 * (2 * 8 + 5) + 16 + 4 * EC + 8 * EC;
   int S = (di.max_smem_optin - extra) / stage_bytes;
   if (S > 8) S = 8;
   if (S < 2) return kErrUnsupported;
+  a.S = S;
   const int smem = S * stage_bytes + extra;
-  const int ntiles = static_cast<int>((T + kBM - 1) / kBM);
+  const int ntiles = (a.T + kBM - 1) / kBM;
   const int grid = ntiles < di.sm_count ? ntiles : di.sm_count;
-  if (cudaFuncSetAttribute(router_gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+  if (cudaFuncSetAttribute(router_gemm_kernel<EC, KP1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
       cudaSuccess)
     return kErrCuda;
-  router_gemm_kernel<<<grid, 192, smem, s>>>(tmx, tmw, z, static_cast<int>(T), d, E, S, err);
+  router_gemm_kernel<EC, KP1><<<grid, 192, smem, s>>>(tmx, tmw, a);
   return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+}
+
+}  // namespace
+
+int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, uint16_t* z,
+                       int32_t* err, cudaStream_t s) {
+  GemmArgs a{z, static_cast<int>(T), d, E, 0, err, nullptr, 0, nullptr, 0, nullptr, nullptr, nullptr};
+  return launch_gemm<0, 1>(x, W, a, s);
+}
+
+int launch_router_route(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, int K, const float* b,
+                        const int64_t* off, int M, uint16_t* z, int32_t* idx, float* tau, int32_t* loads,
+                        int32_t* err, cudaStream_t s) {
+  GemmArgs a{z, static_cast<int>(T), d, E, 0, err, b, K, off, M, idx, tau, loads};
+  if (E == 64) return K + 1 <= 3 ? launch_gemm<64, 3>(x, W, a, s) : launch_gemm<64, 9>(x, W, a, s);
+  if (E == 128) return K + 1 <= 3 ? launch_gemm<128, 3>(x, W, a, s) : launch_gemm<128, 9>(x, W, a, s);
+  return kErrUnsupported;
 }
 
 }  // namespace eqb

@@ -4,6 +4,8 @@
 // Order of work, as in the paper: routing (Sec. 2), Algorithm 1's coarse
 // pass, selection, fine pass, selection and the Eq. (2) bias update, then
 // Load-Error Injection (Sec. 4, Eqs. LEI and norm).  All on one stream.
+// eqb_router_layer_step starts one step earlier, at the router projection
+// (Eq. 1), and routes from the projection's accumulators where it can.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -51,11 +53,16 @@ size_t eqb_layer_workspace_bytes(int32_t E) {
   return carve(nullptr, E, &w);
 }
 
-eqb_status eqb_layer_step(const eqb_bf16* z, const float* b, int64_t T, int32_t E, int32_t K,
-                          const int64_t* mb_offsets, const int64_t* mb_offsets_host, int32_t M,
-                          int64_t r, int32_t* topk_idx, float* tau, int32_t* loads, float* b_next,
-                          float* grad_s, float eta, float c, void* workspace, size_t workspace_bytes,
-                          int32_t* err_flag, void* stream) {
+}  // extern "C"
+
+namespace {
+
+// Checks shared by both step entry points; carves the workspace into w.
+eqb_status check_step(const eqb_bf16* z, const float* b, int64_t T, int32_t E, int32_t K,
+                      const int64_t* mb_offsets, const int64_t* mb_offsets_host, int32_t M,
+                      int32_t* topk_idx, float* tau, int32_t* loads, float* b_next, float* grad_s,
+                      float eta, float c, void* workspace, size_t workspace_bytes, int32_t* err_flag,
+                      Workspace* w) {
   if (T < 1 || E < 2 || K < 1 || K >= E || M < 1) return EQB_ERR_INVALID_ARG;
   if (E > 256 || (E % 8) != 0 || K + 1 > 32) return EQB_ERR_UNSUPPORTED;
   if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
@@ -65,23 +72,29 @@ eqb_status eqb_layer_step(const eqb_bf16* z, const float* b, int64_t T, int32_t 
       !aligned(tau, 4) || !aligned(loads, 4) || !aligned(b_next, 4) || !aligned(grad_s, 16) ||
       !aligned(workspace, 256) || !aligned(err_flag, 4))
     return EQB_ERR_INVALID_ARG;
-  Workspace w;
-  if (workspace_bytes < carve(workspace, E, &w)) return EQB_ERR_INVALID_ARG;
+  if (workspace_bytes < carve(workspace, E, w)) return EQB_ERR_INVALID_ARG;
   if (mb_offsets_host) {
     if (mb_offsets_host[0] != 0 || mb_offsets_host[M] != T) return EQB_ERR_INVALID_ARG;
     for (int l = 0; l < M; ++l)
       if (mb_offsets_host[l + 1] < mb_offsets_host[l]) return EQB_ERR_INVALID_ARG;
   }
-  if (r <= 0) r = eqb_target_rank(T, E, K);
-  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  return EQB_OK;
+}
 
+eqb_status clear(const Workspace& w, int32_t* loads, int32_t E, int32_t M, cudaStream_t s) {
   if (cudaMemsetAsync(w.H, 0, static_cast<size_t>(E) * 256 * 4, s) != cudaSuccess ||
       cudaMemsetAsync(w.L, 0, static_cast<size_t>(E) * 256 * 4, s) != cudaSuccess ||
       cudaMemsetAsync(loads, 0, static_cast<size_t>(M) * E * 4, s) != cudaSuccess)
     return EQB_ERR_CUDA;
+  return EQB_OK;
+}
 
-  eqb::RouteArgs ra{z, b, T, E, K, mb_offsets, M, 0, topk_idx, tau, loads, err_flag};
-  if (int rc = eqb::launch_route(ra, s)) return st(rc);
+// Everything after routing: Algorithm 1's two passes with their selections,
+// the Eq. (2) bias update and LEI.
+eqb_status after_routing(const Workspace& w, const eqb_bf16* z, int64_t T, int32_t E, int32_t K,
+                         const int64_t* mb_offsets, int32_t M, int64_t r, const float* tau,
+                         const int32_t* loads, float* b_next, float* grad_s, float eta, float c,
+                         int32_t* err_flag, cudaStream_t s) {
   eqb::HistArgs h1{z, tau, T, E, nullptr, w.H, err_flag};
   if (int rc = eqb::launch_hist(h1, 1, s)) return st(rc);
   if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
@@ -94,6 +107,55 @@ eqb_status eqb_layer_step(const eqb_bf16* z, const float* b, int64_t T, int32_t 
     if (int rc = eqb::launch_lei(la, s)) return st(rc);
   }
   return EQB_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+eqb_status eqb_layer_step(const eqb_bf16* z, const float* b, int64_t T, int32_t E, int32_t K,
+                          const int64_t* mb_offsets, const int64_t* mb_offsets_host, int32_t M,
+                          int64_t r, int32_t* topk_idx, float* tau, int32_t* loads, float* b_next,
+                          float* grad_s, float eta, float c, void* workspace, size_t workspace_bytes,
+                          int32_t* err_flag, void* stream) {
+  Workspace w;
+  eqb_status rs = check_step(z, b, T, E, K, mb_offsets, mb_offsets_host, M, topk_idx, tau, loads, b_next,
+                             grad_s, eta, c, workspace, workspace_bytes, err_flag, &w);
+  if (rs != EQB_OK) return rs;
+  if (r <= 0) r = eqb_target_rank(T, E, K);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((rs = clear(w, loads, E, M, s)) != EQB_OK) return rs;
+  eqb::RouteArgs ra{z, b, T, E, K, mb_offsets, M, 0, topk_idx, tau, loads, err_flag};
+  if (int rc = eqb::launch_route(ra, s)) return st(rc);
+  return after_routing(w, z, T, E, K, mb_offsets, M, r, tau, loads, b_next, grad_s, eta, c, err_flag, s);
+}
+
+eqb_status eqb_router_layer_step(const eqb_bf16* x, const eqb_bf16* W_r, int64_t T, int32_t d, int32_t E,
+                                 int32_t K, const float* b, const int64_t* mb_offsets,
+                                 const int64_t* mb_offsets_host, int32_t M, int64_t r, eqb_bf16* z,
+                                 int32_t* topk_idx, float* tau, int32_t* loads, float* b_next,
+                                 float* grad_s, float eta, float c, void* workspace,
+                                 size_t workspace_bytes, int32_t* err_flag, void* stream) {
+  if (!x || !W_r || d < 1) return EQB_ERR_INVALID_ARG;
+  if ((d % 64) != 0 || (E % 16) != 0) return EQB_ERR_UNSUPPORTED;
+  if (!aligned(x, 16) || !aligned(W_r, 16)) return EQB_ERR_INVALID_ARG;
+  Workspace w;
+  eqb_status rs = check_step(z, b, T, E, K, mb_offsets, mb_offsets_host, M, topk_idx, tau, loads, b_next,
+                             grad_s, eta, c, workspace, workspace_bytes, err_flag, &w);
+  if (rs != EQB_OK) return rs;
+  if (r <= 0) r = eqb_target_rank(T, E, K);
+  cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
+  if ((rs = clear(w, loads, E, M, s)) != EQB_OK) return rs;
+  if ((E == 64 || E == 128) && K <= 8) {
+    if (int rc = eqb::launch_router_route(x, W_r, T, d, E, K, b, mb_offsets, M, z, topk_idx, tau, loads,
+                                          err_flag, s))
+      return st(rc);
+  } else {
+    if (int rc = eqb::launch_router_gemm(x, W_r, T, d, E, z, err_flag, s)) return st(rc);
+    eqb::RouteArgs ra{z, b, T, E, K, mb_offsets, M, 0, topk_idx, tau, loads, err_flag};
+    if (int rc = eqb::launch_route(ra, s)) return st(rc);
+  }
+  return after_routing(w, z, T, E, K, mb_offsets, M, r, tau, loads, b_next, grad_s, eta, c, err_flag, s);
 }
 
 }  // extern "C"

@@ -122,6 +122,30 @@ def test_router_logits_rejects(lib):
     assert f(FAKE, FAKE, 0, 4096, 128, FAKE, NULL, NULL) == 0
 
 
+def test_router_route_rejects(lib):
+    f = lib.eqb_router_route
+
+    def call(x=FAKE, T=10, d=4096, E=128, K=8, b=FAKE, off=FAKE, M=1, z=FAKE, idx=FAKE, tau=FAKE,
+             loads=FAKE):
+        return f(x, FAKE, T, d, E, K, b, off, M, z, idx, tau, loads, NULL, NULL)
+
+    assert call(E=256) == UNSUPPORTED       # fused routing only for E in {64, 128}
+    assert call(E=96) == UNSUPPORTED
+    assert call(K=9) == UNSUPPORTED         # K + 1 <= 9
+    assert call(d=4000) == UNSUPPORTED      # d not a multiple of 64
+    assert call(K=0) == INVALID
+    assert call(E=64, K=64) == INVALID
+    assert call(x=NULL) == INVALID
+    assert call(b=NULL) == INVALID
+    assert call(tau=NULL) == INVALID
+    assert call(off=NULL) == INVALID        # loads without offsets
+    assert call(M=0) == INVALID
+    assert call(x=MISALIGNED) == INVALID
+    assert call(T=-1) == INVALID
+    assert call(T=0) == 0
+    assert call(T=0, off=NULL, loads=NULL, idx=NULL) == 0
+
+
 def test_layer_step_workspace_size(lib):
     assert lib.eqb_layer_workspace_bytes(256) >= 2 * 256 * 256 * 4 + 256 * 7
     assert lib.eqb_layer_workspace_bytes(256) % 256 == 0
@@ -149,3 +173,25 @@ def test_layer_step_rejects(lib):
     assert call(z=NULL) == INVALID
     assert call(T=0) == INVALID
     assert call(E=60) == UNSUPPORTED
+
+
+def test_router_layer_step_rejects(lib):
+    import numpy as np
+    f = lib.eqb_router_layer_step
+    ws = lib.eqb_layer_workspace_bytes(128)
+    good = np.array([0, 40, 100], np.int64)
+    bad = np.array([0, 60, 50], np.int64)
+    fl = ctypes.c_float(0.0)
+
+    def call(x=FAKE, T=100, d=4096, E=128, K=8, off_h=good, ws_bytes=ws, z=FAKE, M=2):
+        hp = None if off_h is None else off_h.ctypes.data_as(ctypes.c_void_p)
+        return f(x, FAKE, T, d, E, K, FAKE, FAKE, hp, M, 0, z, FAKE, FAKE, FAKE, FAKE, NULL, fl, fl,
+                 FAKE, ws_bytes, NULL, NULL)
+    assert call(x=NULL) == INVALID
+    assert call(x=MISALIGNED) == INVALID
+    assert call(d=4000) == UNSUPPORTED         # d not a multiple of 64
+    assert call(E=72) == UNSUPPORTED           # E not a multiple of 16
+    assert call(off_h=bad) == INVALID
+    assert call(ws_bytes=ws - 1) == INVALID
+    assert call(z=NULL) == INVALID
+    assert call(K=0) == INVALID
