@@ -95,6 +95,18 @@ __device__ __forceinline__ uint32_t hmax2_nan_bf16(uint32_t a, uint32_t b) {
   return r;
 }
 
+// max / min per half (a NaN half loses to a number).
+__device__ __forceinline__ uint32_t hmax2_bf16(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("max.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+__device__ __forceinline__ uint32_t hmin2_bf16(uint32_t a, uint32_t b) {
+  uint32_t r;
+  asm("min.bf16x2 %0, %1, %2;" : "=r"(r) : "r"(a), "r"(b));
+  return r;
+}
+
 // Per half: 0xffff where a >= b, else 0 (NaN compares false).
 __device__ __forceinline__ uint32_t hge2_bf16(uint32_t a, uint32_t b) {
   uint32_t r;
@@ -158,6 +170,55 @@ __device__ __forceinline__ void insert_sorted(float (&v)[KP1], int (&id)[KP1], f
   }
   v[0] = ge[0] ? v[0] : s;
   id[0] = ge[0] ? id[0] : e;
+}
+
+// Bitonic sort of N (a power of two) floats, descending.
+template <int N>
+__device__ __forceinline__ void sort_desc(float (&a)[N]) {
+#pragma unroll
+  for (int k = 2; k <= N; k <<= 1) {
+#pragma unroll
+    for (int j = k >> 1; j > 0; j >>= 1) {
+#pragma unroll
+      for (int i = 0; i < N; ++i) {
+        const int l = i ^ j;
+        if (l > i) {
+          const float x = a[i], y = a[l];
+          const float hi = fmaxf(x, y), lo = fminf(x, y);
+          if ((i & k) == 0) { a[i] = hi; a[l] = lo; } else { a[i] = lo; a[l] = hi; }
+        }
+      }
+    }
+  }
+}
+
+// Bitonic sort, descending, of two independent N-element sequences packed
+// as bf16 pairs: the low halves of a[0..N-1] form one, the high halves the
+// other.  N is a power of two.
+template <int N>
+__device__ __forceinline__ void sort_desc_bf16x2(uint32_t (&a)[N]) {
+#pragma unroll
+  for (int k = 2; k <= N; k <<= 1) {
+#pragma unroll
+    for (int j = k >> 1; j > 0; j >>= 1) {
+#pragma unroll
+      for (int i = 0; i < N; ++i) {
+        const int l = i ^ j;
+        if (l > i) {
+          const uint32_t hi = hmax2_bf16(a[i], a[l]), lo = hmin2_bf16(a[i], a[l]);
+          if ((i & k) == 0) { a[i] = hi; a[l] = lo; } else { a[i] = lo; a[l] = hi; }
+        }
+      }
+    }
+  }
+}
+
+// bf16 pattern `steps` representable values below x (toward -inf), clamped
+// at -inf.  Works on the order-preserving key.
+__device__ __forceinline__ uint32_t bf16_steps_down(uint32_t x, uint32_t steps) {
+  const uint32_t k = kappa16(x);
+  const uint32_t kmin = 0x0080u + steps;  // key of -max_finite is 0x0080
+  return k >= kmin ? kappa16_inv(k - steps) : 0xff80u;
 }
 
 }  // namespace eqb

@@ -61,6 +61,8 @@ struct LeiArgs {
 };
 
 int launch_route(const RouteArgs& a, cudaStream_t s);
+bool route_wide_supported(int E, int K);
+int launch_route_wide(const RouteArgs& a, cudaStream_t s);
 int launch_hist(const HistArgs& a, int pass, cudaStream_t s);
 int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, int32_t* rho,
                   uint16_t* q_hat, int32_t* err, cudaStream_t s);

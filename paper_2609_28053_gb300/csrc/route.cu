@@ -47,33 +47,6 @@ __host__ __device__ inline int warp_region_bytes(int E, int nbuf) {
   return align16(nbuf * 32 * row_stride_bytes(E) + kEntries * 32 * 2 + 4 * E);
 }
 
-template <int N>
-__device__ __forceinline__ void sort_desc(float (&a)[N]) {
-#pragma unroll
-  for (int k = 2; k <= N; k <<= 1) {
-#pragma unroll
-    for (int j = k >> 1; j > 0; j >>= 1) {
-#pragma unroll
-      for (int i = 0; i < N; ++i) {
-        const int l = i ^ j;
-        if (l > i) {
-          const float x = a[i], y = a[l];
-          const float hi = fmaxf(x, y), lo = fminf(x, y);
-          if ((i & k) == 0) { a[i] = hi; a[l] = lo; } else { a[i] = lo; a[l] = hi; }
-        }
-      }
-    }
-  }
-}
-
-// bf16 pattern `steps` representable values below x (toward -inf), clamped
-// at -inf.  Works on the order-preserving key.
-__device__ __forceinline__ uint32_t bf16_steps_down(uint32_t x, uint32_t steps) {
-  const uint32_t k = kappa16(x);
-  const uint32_t kmin = 0x0080u + steps;  // key of -max_finite is 0x0080
-  return k >= kmin ? kappa16_inv(k - steps) : 0xff80u;
-}
-
 template <int KP1, int G>
 __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_per_warp, int nbuf) {
   extern __shared__ __align__(16) uint8_t smem[];
@@ -346,6 +319,7 @@ int launch_route_kp1(const RouteArgs& a, cudaStream_t s) {
 }  // namespace
 
 int launch_route(const RouteArgs& a, cudaStream_t s) {
+  if (route_wide_supported(a.E, a.K)) return launch_route_wide(a, s);
   const int kp1 = a.K + 1;
   if (kp1 <= 2) return launch_route_kp1<2>(a, s);
   if (kp1 <= 3) return launch_route_kp1<3>(a, s);

@@ -58,7 +58,7 @@ def test_forward_small_shapes(T, E, K):
     assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
 
 
-@pytest.mark.parametrize("E,K", [(8, 2), (64, 8), (256, 8), (256, 20)])
+@pytest.mark.parametrize("E,K", [(8, 2), (64, 8), (128, 2), (128, 8), (256, 8), (256, 15), (256, 20)])
 def test_forward_exact_ties(E, K):
     """Integer-valued logits with b = 0: most scores tie, so the candidate
     lists overflow and the exact fallback decides by lower index."""
@@ -67,8 +67,9 @@ def test_forward_exact_ties(E, K):
     assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
 
 
-def test_forward_constant_rows():
-    T, E, K = 300, 64, 8
+@pytest.mark.parametrize("E", [64, 128, 256])
+def test_forward_constant_rows(E):
+    T, K = 300, 8
     z = np.full((T, E), brute.bf16_bits_from_f32(np.float32([0.75]))[0], np.uint16)
     z[::7] = brute.bf16_bits_from_f32(np.float32([-1.5]))[0]
     b = np.zeros(E, np.float32)
@@ -76,9 +77,10 @@ def test_forward_constant_rows():
     assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
 
 
-def test_forward_signed_zero_subnormal_and_large_values():
-    rng = np.random.default_rng(5)
-    T, E, K = 777, 64, 8
+@pytest.mark.parametrize("E", [64, 128, 256])
+def test_forward_signed_zero_subnormal_and_large_values(E):
+    rng = np.random.default_rng(5 + E)
+    T, K = 777, 8
     v = (rng.standard_normal((T, E))).astype(np.float32)
     v[rng.random((T, E)) < 0.1] = 0.0
     v[rng.random((T, E)) < 0.1] = -0.0
