@@ -17,8 +17,8 @@
 //      moved down two bf16 steps, it is <= tau_t; two more steps give the
 //      filter threshold.
 //   B. per-chunk masks of U_e = bf16(z_e + RU(b_e)) >= threshold, every one
-//      of the experts with s_e >= tau_t among them; chunks with a hit are
-//      listed (written unconditionally, the count advances on a hit).
+//      of the experts with s_e >= tau_t among them, kept in shared memory,
+//      with a 32-bit set of the chunks that have a hit.
 //   C. the listed experts, in ascending index, are inserted into a sorted
 //      (K+1)-list by their exact fp32 score s_e = fp32(z_e) + b_e; a new
 //      element goes after equal scores, so ties keep the lower index first.
@@ -82,14 +82,23 @@ struct WideLayout {
   static constexpr int NCH = E / 8;              // 16-byte chunks per row
   static constexpr int RS = wide_row_stride(E);  // staged row stride, bytes
   static constexpr int TILE = 32 * RS;
-  static constexpr int ENT = 32 * NCH * 2;       // listed chunks, u16 per lane and slot
+  static constexpr int ENT = 32 * (NCH / 4) * 4;  // chunk masks, four per word, per lane
   static constexpr int WL = 4 * E;               // load counters
   static constexpr int WARP = (TILE + ENT + WL + 8 + 15) & ~15;  // + the mbarrier
   static constexpr int HEAD = 4 * E + 2 * (2 * E);               // b, RD(b), RU(b)
 };
 
+// Warps per block: as many as shared memory holds (12 at E = 256), at most 16.
+template <int E>
+constexpr int wide_max_warps() {
+  return (232448 - WideLayout<E>::HEAD) / WideLayout<E>::WARP < 16
+             ? (232448 - WideLayout<E>::HEAD) / WideLayout<E>::WARP
+             : 16;
+}
+
 template <int E, int KP1>
-__global__ void __launch_bounds__(512, 1) route_wide_kernel(RouteArgs a, int64_t tiles_per_warp) {
+__global__ void __launch_bounds__(32 * wide_max_warps<E>(), 1)
+    route_wide_kernel(RouteArgs a, int64_t tiles_per_warp) {
   using L = WideLayout<E>;
   constexpr int NCH = L::NCH, NH = NCH / 2;
   extern __shared__ __align__(16) uint8_t smem[];
@@ -102,7 +111,7 @@ __global__ void __launch_bounds__(512, 1) route_wide_kernel(RouteArgs a, int64_t
   uint32_t* bup = bdn + E / 2;                                 // RU(b) packed pairs
   uint8_t* wreg = smem + L::HEAD + wid * L::WARP;
   uint8_t* tile = wreg;
-  uint16_t* ent = reinterpret_cast<uint16_t*>(wreg + L::TILE);
+  uint32_t* mw = reinterpret_cast<uint32_t*>(wreg + L::TILE);  // [NCH/4][32 lanes]
   int* wl = reinterpret_cast<int*>(wreg + L::TILE + L::ENT);
   const uint32_t bar = saddr(wreg + L::TILE + L::ENT + L::WL);
 
@@ -211,55 +220,62 @@ __global__ void __launch_bounds__(512, 1) route_wide_kernel(RouteArgs a, int64_t
     const uint32_t thf = bf16_steps_down(__float_as_uint(theta) >> 16, 4u);
     const uint32_t thf2 = thf | (thf << 16);
 
-    // ---- B: per-chunk masks of U >= threshold, listed in ascending chunk order
-    int cnt = 0;
+    // ---- B: per-chunk masks of U >= threshold, stored four to a word, and
+    // the set of chunks with a hit as one bit per chunk
+    uint32_t hits = 0u;
 #pragma unroll
-    for (int c = 0; c < NCH; ++c) {
-      const uint4 w = lds128(rowp + 16 * c);
-      const uint4 bu = bup4[c];
-      const uint32_t r0 = hge2_bf16(hadd2_bf16(w.x, bu.x), thf2);
-      const uint32_t r1 = hge2_bf16(hadd2_bf16(w.y, bu.y), thf2);
-      const uint32_t r2 = hge2_bf16(hadd2_bf16(w.z, bu.z), thf2);
-      const uint32_t r3 = hge2_bf16(hadd2_bf16(w.w, bu.w), thf2);
-      // element 2q -> bit 2q (low half of r_q), element 2q+1 -> bit 16+2q
-      const uint32_t y = (r0 & 0x00010001u) | (r1 & 0x00040004u) | (r2 & 0x00100010u) | (r3 & 0x00400040u);
-      const uint32_t mask = (y | (y >> 15)) & 0xffu;
-      ent[(cnt << 5) | lane] = static_cast<uint16_t>((c << 8) | mask);
-      cnt += mask != 0u ? 1 : 0;
+    for (int k = 0; k < NCH / 4; ++k) {
+      uint32_t word = 0u;
+#pragma unroll
+      for (int u = 0; u < 4; ++u) {
+        const int c = 4 * k + u;
+        const uint4 w = lds128(rowp + 16 * c);
+        const uint4 bu = bup4[c];
+        const uint32_t r0 = hge2_bf16(hadd2_bf16(w.x, bu.x), thf2);
+        const uint32_t r1 = hge2_bf16(hadd2_bf16(w.y, bu.y), thf2);
+        const uint32_t r2 = hge2_bf16(hadd2_bf16(w.z, bu.z), thf2);
+        const uint32_t r3 = hge2_bf16(hadd2_bf16(w.w, bu.w), thf2);
+        // element 2q -> bit 2q (low half of r_q), element 2q+1 -> bit 16+2q
+        const uint32_t y = (r0 & 0x00010001u) | (r1 & 0x00040004u) | (r2 & 0x00100010u) | (r3 & 0x00400040u);
+        word |= ((y | (y >> 15)) & 0xffu) << (8 * u);
+      }
+      mw[(k << 5) | lane] = word;
+      // high bit of every non-zero byte, then those four bits gathered into
+      // bits 28..31 by one multiply (the partial products do not overlap)
+      const uint32_t nz = (((word & 0x7f7f7f7fu) + 0x7f7f7f7fu) | word) & 0x80808080u;
+      hits |= ((nz * 0x00204081u) >> 28) << (4 * k);
     }
 
-    // ---- C: exact top-(K+1) of the listed experts, one per lane per step,
-    // the next candidate's z and b read one step ahead
+    // ---- C: exact top-(K+1) of the experts with a hit, in ascending index,
+    // one per lane per step; the next candidate's z and b are read one step
+    // ahead.  Refills are branch-free, and a lane that is done inserts -inf,
+    // which leaves its list unchanged.
     float v[KP1];
     int id[KP1];
 #pragma unroll
     for (int j = 0; j < KP1; ++j) { v[j] = -INFINITY; id[j] = 0; }
-    int ei = 0, cb = 0;
+    int cb = 0;
     uint32_t m = 0u;
     auto fetch = [&]() -> int {
-      if (m == 0u && ei < cnt) {
-        const uint32_t en = ent[(ei << 5) | lane];
-        cb = static_cast<int>(en >> 8) << 3;
-        m = en & 0xffu;
-        ++ei;
-      }
-      if (m == 0u) return -1;
-      const int e = cb + __ffs(m) - 1;
+      const bool need = m == 0u && hits != 0u;
+      const int c = __ffs(hits) - 1;
+      const int cc = need ? c : 0;
+      const uint32_t word = mw[((cc >> 2) << 5) | lane];
+      m = need ? (word >> ((cc & 3) << 3)) & 0xffu : m;
+      cb = need ? c << 3 : cb;
+      hits = need ? hits & (hits - 1u) : hits;
+      const int e = m != 0u ? cb + __ffs(m) - 1 : -1;
       m &= m - 1u;
       return e;
     };
     int e0 = fetch();
-    uint32_t z0 = e0 >= 0 ? lds_u16(rowp + 2 * e0) : 0u;
-    float b0 = e0 >= 0 ? bs[e0] : 0.f;
+    uint32_t z0 = lds_u16(rowp + 2 * max(e0, 0));
+    float b0 = bs[max(e0, 0)];
     while (__any_sync(kFull, e0 >= 0)) {
       const int e1 = fetch();
-      uint32_t z1 = 0u;
-      float b1 = 0.f;
-      if (e1 >= 0) {
-        z1 = lds_u16(rowp + 2 * e1);
-        b1 = bs[e1];
-      }
-      if (e0 >= 0) insert_sorted<KP1>(v, id, bf16_bits_to_f32(z0) + b0, e0);
+      const uint32_t z1 = lds_u16(rowp + 2 * max(e1, 0));
+      const float b1 = bs[max(e1, 0)];
+      insert_sorted<KP1>(v, id, e0 >= 0 ? bf16_bits_to_f32(z0) + b0 : -INFINITY, e0);
       e0 = e1;
       z0 = z1;
       b0 = b1;
@@ -323,7 +339,7 @@ int launch_wide_t(const RouteArgs& a, cudaStream_t s) {
   DeviceInfo di;
   if (int rc = device_info(&di)) return rc;
   int nw = (di.max_smem_optin - L::HEAD) / L::WARP;
-  if (nw > 16) nw = 16;
+  if (nw > wide_max_warps<E>()) nw = wide_max_warps<E>();
   if (nw < 1) return kErrUnsupported;
   const int smem = L::HEAD + nw * L::WARP;
   int ctas_per_sm = (228 * 1024 - 1024) / (smem + 1024);
