@@ -228,6 +228,20 @@ class Step:
         return d
 
 
+def dram_traffic(path, kernel, T, E):
+    """DRAM bytes (read + write) of one launch of `kernel` at this T and E, as
+    recorded from an ncu capture of the same kernel code (lines of
+    `kernel T E bytes`; '#' starts a comment); None when not recorded."""
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        for line in f:
+            parts = line.split("#", 1)[0].split()
+            if len(parts) == 4 and parts[0] == kernel and int(parts[1]) == T and int(parts[2]) == E:
+                return int(parts[3])
+    return None
+
+
 def cpu_oracle_sample(z_dev, b_dev, g_dev, K, n_tokens, M_per):
     """The oracle, as it stands, on the first n_tokens of the workload:
     routing, the exact quantile of every expert over the sample, the bias
@@ -302,7 +316,7 @@ def main():
     ap.add_argument("--cpu-sample-tokens", type=int, default=131072)
     ap.add_argument("--ref-sample-tokens", type=int, default=32768)
     ap.add_argument("--no-cpu-baseline", action="store_true")
-    ap.add_argument("--traffic-json", default=os.path.join(ROOT, "profiles", "traffic.json"))
+    ap.add_argument("--traffic-file", default=os.path.join(ROOT, "profiles", "dram_traffic_per_launch.txt"))
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
         args.warmup = 3
@@ -377,13 +391,7 @@ def main():
     peak, peak_kind = measured_peaks()
     dom = max(per_kernel, key=per_kernel.get)
     dom_bytes = alg.get(dom)
-    traffic = None
-    if os.path.exists(args.traffic_json):
-        with open(args.traffic_json) as f:
-            tj = json.load(f)
-        ent = tj.get(dom)
-        if ent and ent.get("T") == T and ent.get("E") == E:
-            traffic = ent.get("bytes_per_launch")
+    traffic = dram_traffic(args.traffic_file, dom, T, E)
     achieved = dom_bytes / (per_kernel[dom] * 1e-3) / 1e9
     roofline = {"bound": "hbm", "kernel": dom, "achieved": achieved, "peak": peak, "unit": "GB/s",
                 "frac": achieved / peak, "peak_source": peak_kind, "traffic": traffic,

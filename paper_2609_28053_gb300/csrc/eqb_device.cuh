@@ -28,6 +28,23 @@ __device__ __forceinline__ uint32_t pack_bf16x2_rn(float lo, float hi) {
   return r;
 }
 
+// (t - lo, t - hi) for the two bf16 values of a packed word, as one packed
+// fp32 subtraction (round to nearest even, subnormals kept), rounded to a
+// bf16 pair: the margins of two experts.  tt holds t in both halves.
+__device__ __forceinline__ uint64_t f32x2_splat(float t) {
+  uint64_t r;
+  asm("mov.b64 %0, {%1, %1};" : "=l"(r) : "f"(t));
+  return r;
+}
+__device__ __forceinline__ uint32_t margins_bf16x2(uint64_t tt, uint32_t zw) {
+  uint64_t zz, dd;
+  asm("mov.b64 %0, {%1, %2};" : "=l"(zz) : "f"(__uint_as_float(zw << 16)), "f"(__uint_as_float(zw & 0xffff0000u)));
+  asm("sub.rn.f32x2 %0, %1, %2;" : "=l"(dd) : "l"(tt), "l"(zz));
+  float lo, hi;
+  asm("mov.b64 {%0, %1}, %2;" : "=f"(lo), "=f"(hi) : "l"(dd));
+  return pack_bf16x2_rn(lo, hi);
+}
+
 // fp32 max that propagates NaN (used where a NaN must stay visible).
 __device__ __forceinline__ float fmax_nan(float a, float b) {
   float r;

@@ -8,9 +8,9 @@
 // every key; pass 2 counts the low byte of the keys whose high byte is u_e.
 //
 // Work per element is kept to a handful of instructions by working on packed
-// pairs: one 32-bit word of z holds two experts, their two margins are
-// rounded with one cvt.rn.bf16x2, and one PRMT (sign replicate) plus one LOP3
-// give both internal keys (kappa ^ 0x8000, so the stored high byte is the
+// pairs: one 32-bit word of z holds two experts, their two fp32 differences
+// are one packed f32x2 subtraction, rounded with one cvt.rn.bf16x2, and one
+// PRMT (sign replicate) plus one LOP3 give both internal keys (kappa ^ 0x8000, so the stored high byte is the
 // true one ^ 0x80 and is translated back at the flush).
 //
 // Bins: a CTA owns ET experts (all E when E <= 256 is a power of two) and
@@ -77,9 +77,10 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
 
   auto process = [&](const uint4& w4, float tv) {
     const uint32_t zw[4] = {w4.x, w4.y, w4.z, w4.w};
+    const uint64_t tt = f32x2_splat(tv);
 #pragma unroll
     for (int p = 0; p < 4; ++p) {
-      const uint32_t m = pack_bf16x2_rn(tv - bf16_lo(zw[p]), tv - bf16_hi(zw[p]));
+      const uint32_t m = margins_bf16x2(tt, zw[p]);
       const uint32_t k = kappa2_internal(m);
       const uint32_t row = base + 1024u * p;
       if (PASS == 1) {
