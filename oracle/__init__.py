@@ -70,6 +70,7 @@ def _load():
                 "oracle_bias_update": [P, i32, P],
                 "oracle_lei": [P, P, P, i32, i64, i32, i32, f32, f32, P, P],
                 "oracle_router_logits": [P, P, i64, i32, i32, P, i64, P, P],
+                "oracle_maxvio": [P, P, i32, i32, i32, P, P, P],
             }
             for name, args in sig.items():
                 fn = getattr(lib, name)
@@ -264,6 +265,21 @@ def router_logits(x_bits, W_bits, rows):
     _check(_load().oracle_router_logits(_ptr(x_bits), _ptr(W_bits), T, d, E, _ptr(rows), len(rows),
                                         _ptr(out), _ptr(ab)), "oracle_router_logits")
     return out, ab
+
+
+def maxvio(loads, offsets, K):
+    """Sec. 5 / App. E: MaxVio = max_e [f_e / fbar - 1], fbar = K|B|/E, for the
+    loads summed over the step (global) and per non-empty microbatch, then
+    averaged (local).  Returns (global, local, per_microbatch float64 [M])."""
+    loads = _c(loads, np.int32)
+    M, E = loads.shape
+    offsets = _c(offsets, np.int64)
+    g = ctypes.c_double(0.0)
+    lo = ctypes.c_double(0.0)
+    per = np.zeros(M, np.float64)
+    _check(_load().oracle_maxvio(_ptr(loads), _ptr(offsets), M, E, K, ctypes.byref(g),
+                                 ctypes.byref(lo), _ptr(per)), "oracle_maxvio")
+    return g.value, lo.value, per
 
 
 def eqb_step(z_bits, b, K, offsets=None):

@@ -19,6 +19,8 @@
  *   bias update  Eq. (2) centering b = b_hat - mean(b_hat).
  *   LEI          Sec. 4, Eq. (LEI) and Eq. (norm).
  *   router       Sec. 2: z_t = W_r x_t, the dot products in fp64.
+ *   MaxVio       Sec. 5 (Metrics) and App. E (balance metrics):
+ *                max_e [f_e(B) / fbar(B) - 1], global and local.
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - scores s = fp32(z) + b in fp32 round-to-nearest-even; tau is fp32;
@@ -34,7 +36,10 @@
  *   - LEI adds eta * rho~_e to every (t, e) of the local batch (selected or
  *     not), one shared scale per microbatch, c <= 0 meaning unnormalised;
  *     the injected term and the sum are formed in fp64 and rounded to fp32
- *     once.
+ *     once;
+ *   - MaxVio in fp64 with fbar = K * |B| / E; Local MaxVio is the plain mean
+ *     over the non-empty microbatches (an empty one has no fbar), summed in
+ *     ascending microbatch order.
  *
  * Compile with -ffp-contract=off and without -ffast-math.
  */
@@ -358,5 +363,48 @@ int oracle_router_logits(const uint16_t *x, const uint16_t *W, int64_t T, int32_
       if (abs_out) abs_out[i * E + e] = acc_abs;
     }
   }
+  return ORACLE_OK;
+}
+
+/* ---- balance metric: Sec. 5 (Metrics), App. E --------------------------- */
+
+/* MaxVio(B) = max_e [ f_e(B) / fbar(B) - 1 ], fbar(B) = K |B| / E, in fp64.
+ *   global   loads summed over all microbatches, |B| = T = off[M];
+ *   local    MaxVio of every non-empty microbatch l (|B| = off[l+1] - off[l])
+ *            and their plain mean, summed in ascending l; per_mb (optional,
+ *            [M]) receives each microbatch's value (0 for an empty one).
+ * Returns ORACLE_ERR_ARG when every microbatch is empty. */
+int oracle_maxvio(const int32_t *loads, const int64_t *off, int32_t M, int32_t E, int32_t K,
+                  double *global, double *local, double *per_mb) {
+  if (E < 1 || K < 1 || M < 1 || off == NULL || off[0] != 0) return ORACLE_ERR_ARG;
+  int64_t T = off[M];
+  if (T < 1 || !check_offsets(off, M, T)) return ORACLE_ERR_ARG;
+  double sum = 0.0;
+  int32_t count = 0;
+  for (int32_t l = 0; l < M; ++l) {
+    int64_t n = off[l + 1] - off[l];
+    double v = 0.0;
+    if (n > 0) {
+      const double fbar_l = (double)K * (double)n / (double)E;
+      v = -INFINITY;
+      for (int32_t e = 0; e < E; ++e) {
+        double x = (double)loads[(int64_t)l * E + e] / fbar_l - 1.0;
+        if (x > v) v = x;
+      }
+      sum += v;
+      ++count;
+    }
+    if (per_mb) per_mb[l] = v;
+  }
+  double fbar = (double)K * (double)T / (double)E;
+  double g = -INFINITY;
+  for (int32_t e = 0; e < E; ++e) {
+    int64_t f = 0;
+    for (int32_t l = 0; l < M; ++l) f += loads[(int64_t)l * E + e];
+    double x = (double)f / fbar - 1.0;
+    if (x > g) g = x;
+  }
+  *global = g;
+  *local = sum / (double)count;
   return ORACLE_OK;
 }

@@ -31,6 +31,10 @@ MUTANTS = {
     "rho_off_by_one": ("rho[e] = (int32_t)(r - below);", "rho[e] = (int32_t)(r - below + 1);"),
     "loads_ignore_microbatch": ("loads[(int64_t)l * E + buf[k].e] += 1;", "loads[buf[k].e] += 1;"),
     "score_drops_bias": ("buf[e].s = zf + b[e];", "buf[e].s = zf;"),
+    "maxvio_local_counts_empty": ("*local = sum / (double)count;", "*local = sum / (double)M;"),
+    "maxvio_drops_K": ("const double fbar_l = (double)K * (double)n / (double)E;",
+                       "const double fbar_l = (double)n / (double)E;"),
+    "maxvio_global_is_max_local": ("  *global = g;", "  *global = sum > g ? sum : g;"),
     "lei_not_all_experts": ("for (int32_t e = 0; e < E; ++e)\n          g_out[t * E + e] = (float)((double)g[t * E + e] + a[e]);",
                             "for (int32_t e = 0; e < E; ++e)\n          g_out[t * E + e] = (loads[(int64_t)l * E + e] > 0) ? (float)((double)g[t * E + e] + a[e]) : g[t * E + e];"),
 }

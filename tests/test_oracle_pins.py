@@ -214,6 +214,8 @@ def test_cyclic_balanced_assignment_golden():
         g_out, a = oracle.lei(g, st["loads"], off, K, eta=0.5, c=1.0)
         assert np.all(a == c["lei_coefficient"])
         assert np.array_equal(g_out, g)
+        mg, ml, _ = oracle.maxvio(st["loads"], off, K)
+        assert (mg, ml) == (c["maxvio_global"], c["maxvio_local"])
 
 
 def test_constant_columns_closed_form():
@@ -337,3 +339,64 @@ def test_router_logits_matches_float64_matmul_and_one_hot():
     np.fill_diagonal(onehot, 1.0)
     zo, _ = oracle.router_logits(brute.bf16_bits_from_f32(onehot), W, np.arange(0, d, 7))
     assert np.array_equal(zo, Wf[:, ::7].T)
+
+
+# ------------------------------------------------------------------ MaxVio
+
+def test_maxvio_paper_example():
+    """Sec. 5 / App. E: a Local MaxVio of 5.96 means the most-loaded expert
+    receives 6.96 times its uniform load.  E = 100, K = 4, n = 2500 tokens:
+    the uniform load is K n / E = 100, so a top load of 696 gives 5.96."""
+    E, K, n = 100, 4, 2500
+    loads = np.full((1, E), 94, np.int32)
+    loads[0, 0] = 696
+    loads[0, E - 1] = K * n - 696 - 94 * (E - 2)  # loads sum to K n
+    assert loads.sum() == K * n and 0 <= loads.min() and loads[0, 1:].max() < 696
+    g, l, per = oracle.maxvio(loads, np.array([0, n]), K)
+    assert g == l == per[0] == pytest.approx(5.96, abs=1e-12)
+
+
+def test_maxvio_all_tokens_on_one_expert():
+    """Every token of a microbatch picks expert 3: its load is n = fbar E / K,
+    so MaxVio = E/K - 1 for that microbatch."""
+    E, K = 16, 4
+    off = np.array([0, 40, 40, 100], np.int64)  # the middle microbatch is empty
+    loads = np.zeros((3, E), np.int32)
+    for l, n in enumerate(np.diff(off)):
+        loads[l, 3] = n
+        loads[l, 4:4 + K - 1] = n
+    g, loc, per = oracle.maxvio(loads, off, K)
+    assert per[0] == per[2] == E / K - 1 and per[1] == 0.0
+    assert loc == E / K - 1
+    assert g == E / K - 1
+
+
+@pytest.mark.parametrize("seed", range(4))
+def test_maxvio_against_exact_rationals(seed):
+    """Random loads over uneven (one empty) microbatches: the definition
+    evaluated in exact rationals, max over experts of f_e / fbar - 1 with
+    fbar = K |B| / E; Local is the plain mean over the non-empty microbatches
+    and Global uses the loads summed over the step."""
+    from fractions import Fraction
+    rng = np.random.default_rng(seed)
+    E, K, M = 24, 3, 5
+    off = np.sort(np.concatenate([[0], rng.integers(1, 400, M - 1), [400]])).astype(np.int64)
+    off[2] = off[1]  # an empty microbatch
+    loads = np.zeros((M, E), np.int32)
+    for l in range(M):
+        n = int(off[l + 1] - off[l])
+        for _ in range(n):
+            loads[l, rng.choice(E, K, replace=False, p=rng.dirichlet(np.ones(E)))] += 1
+    g, loc, per = oracle.maxvio(loads, off, K)
+    exact = []
+    for l in range(M):
+        n = int(off[l + 1] - off[l])
+        if n:
+            fbar = Fraction(K * n, E)
+            exact.append(max(Fraction(int(f)) / fbar - 1 for f in loads[l]))
+    want_local = sum(exact, Fraction(0)) / len(exact)
+    fbar_g = Fraction(K * int(off[-1]), E)
+    want_global = max(Fraction(int(f)) / fbar_g - 1 for f in loads.sum(0))
+    assert abs(Fraction(loc) - want_local) <= Fraction(1, 2 ** 48)
+    assert abs(Fraction(g) - want_global) <= Fraction(1, 2 ** 48)
+    assert per[1] == 0.0
