@@ -221,6 +221,26 @@ eqb_status eqb_layer_step_noalloc(const eqb_bf16 *z, const float *b, int64_t T, 
 eqb_status eqb_router_logits(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t T, int32_t d,
                              int32_t E, eqb_bf16 *z, int32_t *err_flag, void *stream);
 
+/* Balance metric MaxVio, Sec. 5 (Metrics) and App. E (balance metrics):
+ *   MaxVio(B) = max_e [ f_e(B) / fbar(B) - 1 ],   fbar(B) = K |B| / E,
+ * in fp64 (fbar formed as (K * |B|) / E, then one division and one
+ * subtraction).
+ *   maxvio[0]  Global MaxVio: the loads summed over the M microbatches,
+ *              |B| = offsets[M] - offsets[0].
+ *   maxvio[1]  Local MaxVio: the plain mean, summed in ascending order, of
+ *              the per-microbatch values over the non-empty microbatches (an
+ *              empty one has no fbar); 0 if every microbatch is empty.
+ *   loads      device int32 [M,E] (in): per-microbatch loads, as written by
+ *              eqb_route_topk or eqb_layer_step
+ *   mb_offsets device int64 [M+1] (in): as in eqb_route_topk
+ *   maxvio     device double [2] (out), 8-byte aligned
+ *   per_mb     device double [M] (out, nullable): each microbatch's MaxVio,
+ *              0 for an empty one
+ * The paper reports the maximum over layers and a mean over steps; a caller
+ * takes those across calls.  Supported: 1 <= M <= 16384. */
+eqb_status eqb_maxvio(const int32_t *loads, const int64_t *mb_offsets, int32_t M, int32_t E,
+                      int32_t K, double *maxvio, double *per_mb, void *stream);
+
 /* Router logits and routing in one kernel: eqb_router_logits followed by
  * eqb_route_topk (without hist_hi), with each token routed straight from the
  * tensor-memory accumulator of its row, so z is written once and not read

@@ -71,6 +71,7 @@ def _load():
                 "oracle_lei": [P, P, P, i32, i64, i32, i32, f32, f32, P, P],
                 "oracle_router_logits": [P, P, i64, i32, i32, P, i64, P, P],
                 "oracle_maxvio": [P, P, i32, i32, i32, P, P, P],
+                "oracle_gshard": [P, P, P, P, i32, i64, i32, i32, f32, P],
             }
             for name, args in sig.items():
                 fn = getattr(lib, name)
@@ -280,6 +281,21 @@ def maxvio(loads, offsets, K):
     _check(_load().oracle_maxvio(_ptr(loads), _ptr(offsets), M, E, K, ctypes.byref(g),
                                  ctypes.byref(lo), _ptr(per)), "oracle_maxvio")
     return g.value, lo.value, per
+
+
+def gshard(g, z_bits, loads, offsets, K, alpha):
+    """App. D, Eq. (gshard-grad): g + alpha * d/ds sum_e F_e P^G_e per local
+    batch, with s = sigmoid(z), F stop-gradient.  Returns float32 [T,E]."""
+    g = _c(g, np.float32)
+    z_bits = _c(z_bits, np.uint16)
+    T, E = z_bits.shape
+    loads = _c(loads, np.int32)
+    offsets = _c(offsets, np.int64)
+    M = len(offsets) - 1
+    out = g.copy()
+    _check(_load().oracle_gshard(_ptr(g), _ptr(z_bits), _ptr(loads), _ptr(offsets), M, T, E, K,
+                                 float(alpha), _ptr(out)), "oracle_gshard")
+    return out
 
 
 def eqb_step(z_bits, b, K, offsets=None):

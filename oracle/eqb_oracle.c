@@ -21,6 +21,8 @@
  *   router       Sec. 2: z_t = W_r x_t, the dot products in fp64.
  *   MaxVio       Sec. 5 (Metrics) and App. E (balance metrics):
  *                max_e [f_e(B) / fbar(B) - 1], global and local.
+ *   GShard STE   App. D, Eq. (gshard-grad): the gradient of the GShard
+ *                auxiliary loss (Sec. 2) with respect to the router scores.
  *
  * Readings where the paper is silent (each also listed in the design notes):
  *   - scores s = fp32(z) + b in fp32 round-to-nearest-even; tau is fp32;
@@ -39,7 +41,11 @@
  *     once;
  *   - MaxVio in fp64 with fbar = K * |B| / E; Local MaxVio is the plain mean
  *     over the non-empty microbatches (an empty one has no fbar), summed in
- *     ascending microbatch order.
+ *     ascending microbatch order;
+ *   - GShard: the router scores are s = sigmoid(fp32(z)) of the unbiased
+ *     logits (Sec. 2), the batch of P^G is the local microbatch, and the
+ *     injected term is alpha times the gradient of sum_e F_e P^G_e (the
+ *     auxiliary loss), formed in fp64 and added to g with one rounding.
  *
  * Compile with -ffp-contract=off and without -ffast-math.
  */
@@ -406,5 +412,45 @@ int oracle_maxvio(const int32_t *loads, const int64_t *off, int32_t M, int32_t E
   }
   *global = g;
   *local = sum / (double)count;
+  return ORACLE_OK;
+}
+
+/* ---- GShard auxiliary-loss gradient: App. D, Eq. (gshard-grad) ---------- */
+
+/* For microbatch l with n tokens and loads f_e:  F_e = f_e / (K n),
+ * R_e = F_e - 1/E; for each of its tokens t, with s_e = sigmoid(z_{t,e}),
+ * d_t = sum_e s_e and p_e = s_e / d_t,
+ *   g_out[t, j] = fp32( g[t, j] + alpha / (n d_t) * (R_j - sum_e p_e R_e) ),
+ * all in fp64.  Empty microbatches have no tokens. */
+int oracle_gshard(const float *g, const uint16_t *z, const int32_t *loads, const int64_t *off,
+                  int32_t M, int64_t T, int32_t E, int32_t K, float alpha, float *g_out) {
+  if (T < 0 || E < 1 || K < 1 || !check_offsets(off, M, T)) return ORACLE_ERR_ARG;
+  double *R = (double *)malloc(sizeof(double) * (size_t)E);
+  double *s = (double *)malloc(sizeof(double) * (size_t)E);
+  if (!R || !s) {
+    free(R);
+    free(s);
+    return ORACLE_ERR_NOMEM;
+  }
+  for (int32_t l = 0; l < M; ++l) {
+    const int64_t n = off[l + 1] - off[l];
+    if (n == 0) continue;
+    for (int32_t e = 0; e < E; ++e)
+      R[e] = (double)loads[(int64_t)l * E + e] / ((double)K * (double)n) - 1.0 / (double)E;
+    for (int64_t t = off[l]; t < off[l + 1]; ++t) {
+      double d = 0.0;
+      for (int32_t e = 0; e < E; ++e) {
+        s[e] = 1.0 / (1.0 + exp(-(double)bf16_bits_to_f32(z[t * E + e])));
+        d += s[e];
+      }
+      double m = 0.0;
+      for (int32_t e = 0; e < E; ++e) m += (s[e] / d) * R[e];
+      const double scale = (double)alpha / ((double)n * d);
+      for (int32_t j = 0; j < E; ++j)
+        g_out[t * E + j] = (float)((double)g[t * E + j] + scale * (R[j] - m));
+    }
+  }
+  free(R);
+  free(s);
   return ORACLE_OK;
 }

@@ -32,6 +32,7 @@ __all__ = [
     "eqb_margin_hist_pass2", "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad",
     "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route", "eqb_router_layer_step",
+    "eqb_maxvio",
 ]
 
 
@@ -185,6 +186,22 @@ def eqb_router_route(x, W_r, b, K, mb_offsets=None, z=None, topk_idx=None, tau=N
                                    _p(topk_idx), _p(tau), _p(loads), _p(err_flag), _stream(stream)),
            "eqb_router_route")
     return z, topk_idx, tau
+
+
+def eqb_maxvio(loads, mb_offsets, K, out=None, per_mb=None, stream=None):
+    """Global and Local MaxVio (Sec. 5 metrics) of int32 loads [M,E] over the
+    microbatches given by mb_offsets; returns a float64 CUDA tensor [2]
+    (global, local)."""
+    M, E = loads.shape
+    _need(loads, torch.int32, "loads")
+    _need(mb_offsets, torch.int64, "mb_offsets", (M + 1,))
+    if out is None:
+        out = torch.empty(2, dtype=torch.float64, device=loads.device)
+    _need(out, torch.float64, "out", (2,))
+    _need(per_mb, torch.float64, "per_mb", (M,) if per_mb is not None else None)
+    _check(load().eqb_maxvio(_p(loads), _p(mb_offsets), M, E, K, _p(out), _p(per_mb), _stream(stream)),
+           "eqb_maxvio")
+    return out
 
 
 def eqb_layer_workspace_bytes(E: int) -> int:

@@ -183,4 +183,14 @@ eqb_status eqb_router_route(const eqb_bf16* x, const eqb_bf16* W_r, int64_t T, i
                                             err_flag, as_stream(stream)));
 }
 
+eqb_status eqb_maxvio(const int32_t* loads, const int64_t* mb_offsets, int32_t M, int32_t E, int32_t K,
+                      double* maxvio, double* per_mb, void* stream) {
+  if (M < 1 || E < 1 || K < 1) return EQB_ERR_INVALID_ARG;
+  if (M > 16384) return EQB_ERR_UNSUPPORTED;
+  if (!loads || !mb_offsets || !maxvio) return EQB_ERR_INVALID_ARG;
+  if (!aligned(loads, 4) || !aligned(mb_offsets, 8) || !aligned(maxvio, 8) || !aligned(per_mb, 8))
+    return EQB_ERR_INVALID_ARG;
+  return to_status(eqb::launch_maxvio(loads, mb_offsets, M, E, K, maxvio, per_mb, as_stream(stream)));
+}
+
 }  // extern "C"

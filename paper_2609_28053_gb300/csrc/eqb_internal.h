@@ -70,6 +70,8 @@ int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t
 int launch_lei(const LeiArgs& a, cudaStream_t s);
 int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, uint16_t* z,
                        int32_t* err, cudaStream_t s);
+int launch_maxvio(const int32_t* loads, const int64_t* off, int M, int E, int K, double* out, double* per_mb,
+                  cudaStream_t s);
 int launch_router_route(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, int K, const float* b,
                         const int64_t* off, int M, uint16_t* z, int32_t* idx, float* tau, int32_t* loads,
                         int32_t* err, cudaStream_t s);

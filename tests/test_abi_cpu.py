@@ -195,3 +195,13 @@ def test_router_layer_step_rejects(lib):
     assert call(ws_bytes=ws - 1) == INVALID
     assert call(z=NULL) == INVALID
     assert call(K=0) == INVALID
+
+
+def test_maxvio_rejects(lib):
+    f = lib.eqb_maxvio
+    assert f(FAKE, FAKE, 0, 8, 2, FAKE, NULL, NULL) == INVALID
+    assert f(FAKE, FAKE, 16385, 8, 2, FAKE, NULL, NULL) == UNSUPPORTED
+    assert f(NULL, FAKE, 4, 8, 2, FAKE, NULL, NULL) == INVALID
+    assert f(FAKE, FAKE, 4, 8, 2, NULL, NULL, NULL) == INVALID
+    assert f(FAKE, FAKE, 4, 0, 2, FAKE, NULL, NULL) == INVALID
+    assert f(FAKE, FAKE, 4, 8, 2, ctypes.c_void_p(0x10004), NULL, NULL) == INVALID  # maxvio not 8-aligned

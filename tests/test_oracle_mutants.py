@@ -35,6 +35,12 @@ MUTANTS = {
     "maxvio_drops_K": ("const double fbar_l = (double)K * (double)n / (double)E;",
                        "const double fbar_l = (double)n / (double)E;"),
     "maxvio_global_is_max_local": ("  *global = g;", "  *global = sum > g ? sum : g;"),
+    "gshard_drops_mean": ("g_out[t * E + j] = (float)((double)g[t * E + j] + scale * (R[j] - m));",
+                          "g_out[t * E + j] = (float)((double)g[t * E + j] + scale * R[j]);"),
+    "gshard_batch_is_step": ("const double scale = (double)alpha / ((double)n * d);",
+                             "const double scale = (double)alpha / ((double)T * d);"),
+    "gshard_drops_score_sum": ("for (int32_t e = 0; e < E; ++e) m += (s[e] / d) * R[e];",
+                               "for (int32_t e = 0; e < E; ++e) m += s[e] * R[e];"),
     "lei_not_all_experts": ("for (int32_t e = 0; e < E; ++e)\n          g_out[t * E + e] = (float)((double)g[t * E + e] + a[e]);",
                             "for (int32_t e = 0; e < E; ++e)\n          g_out[t * E + e] = (loads[(int64_t)l * E + e] > 0) ? (float)((double)g[t * E + e] + a[e]) : g[t * E + e];"),
 }

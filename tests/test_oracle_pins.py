@@ -400,3 +400,62 @@ def test_maxvio_against_exact_rationals(seed):
     assert abs(Fraction(loc) - want_local) <= Fraction(1, 2 ** 48)
     assert abs(Fraction(g) - want_global) <= Fraction(1, 2 ** 48)
     assert per[1] == 0.0
+
+
+# ------------------------------------------------------------------ GShard STE
+
+def gshard_case(T, E, K, M, seed):
+    rng = np.random.default_rng(seed)
+    z = brute.bf16_bits_from_f32(rng.standard_normal((T, E)).astype(np.float32))
+    off = ragged_offsets(T, M, seed=seed)
+    _, _, loads = oracle.route(z, np.zeros(E, np.float32), K, off)
+    g = (0.1 * rng.standard_normal((T, E))).astype(np.float32)
+    return z, off, loads, g
+
+
+def test_gshard_is_gradient_of_aux_loss():
+    """Finite differences of L = alpha sum_e F_e P^G_e (Sec. 2, the GShard
+    loss with F held fixed), P^G_e = |B_l|^-1 sum_t s_{t,e} / sum_j s_{t,j},
+    with respect to each score s_{t,j}, against the injected term."""
+    T, E, K, M = 6, 5, 2, 2
+    z, _, _, g = gshard_case(T, E, K, M, seed=11)
+    off = np.array([0, 2, 6], np.int64)  # two local batches, neither the whole step
+    _, _, loads = oracle.route(z, np.zeros(E, np.float32), K, off)
+    alpha = 0.75
+    term = oracle.gshard(np.zeros((T, E), np.float32), z, loads, off, K, alpha).astype(np.float64)
+    s0 = 1.0 / (1.0 + np.exp(-brute.f32_from_bf16_bits(z).astype(np.float64)))
+
+    def loss(s):
+        total = 0.0
+        for l in range(M):
+            a, b_ = int(off[l]), int(off[l + 1])
+            if b_ == a:
+                continue
+            F = loads[l] / (K * (b_ - a))
+            P = (s[a:b_] / s[a:b_].sum(1, keepdims=True)).mean(0)
+            total += alpha * float((F * P).sum())
+        return total
+
+    h = 1e-6
+    for t in range(T):
+        for j in range(E):
+            sp, sm = s0.copy(), s0.copy()
+            sp[t, j] += h
+            sm[t, j] -= h
+            fd = (loss(sp) - loss(sm)) / (2 * h)
+            assert abs(fd - term[t, j]) <= 1e-7 + 1e-5 * abs(fd), (t, j, fd, term[t, j])
+
+
+def test_gshard_orthogonal_to_scores_and_zero_when_balanced():
+    """The aux loss depends on s_t only through s_t / sum_j s_t,j, so the
+    gradient is orthogonal to s_t (sum_j s_tj dL/ds_tj = 0); with loads equal
+    to K n / E for every expert (F = Q) the term vanishes and g is unchanged."""
+    T, E, K, M = 200, 8, 2, 3
+    z, off, loads, g = gshard_case(T, E, K, M, seed=5)
+    term = oracle.gshard(np.zeros((T, E), np.float32), z, loads, off, K, 1.0).astype(np.float64)
+    s = 1.0 / (1.0 + np.exp(-brute.f32_from_bf16_bits(z).astype(np.float64)))
+    assert np.max(np.abs((s * term).sum(1))) < 1e-9
+    assert np.max(np.abs(term)) > 1e-6
+    off_b = np.array([0, 80, 160, 200], np.int64)  # K n / E integral: n in {80, 80, 40}
+    bal = np.repeat((K * np.diff(off_b) // E)[:, None], E, axis=1).astype(np.int32)
+    assert np.array_equal(oracle.gshard(g, z, bal, off_b, K, 3.0), g)
