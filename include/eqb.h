@@ -221,6 +221,23 @@ eqb_status eqb_layer_step_noalloc(const eqb_bf16 *z, const float *b, int64_t T, 
 eqb_status eqb_router_logits(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t T, int32_t d,
                              int32_t E, eqb_bf16 *z, int32_t *err_flag, void *stream);
 
+/* GShard auxiliary-loss gradient: the comparison injection beside LEI
+ * (Sec. 2, the loss alpha sum_e F_e P^G_e with F stop-gradient; App. D,
+ * Eq. (gshard-grad)).  For every token t of microbatch l (n_l tokens):
+ *   s_e = sigmoid(fp32(z_{t,e})),  d_t = sum_e s_e,  p_e = s_e / d_t,
+ *   R_e = f_{l,e} / (K n_l) - 1/E,
+ *   grad_s[t, j] += alpha / (n_l d_t) * (R_j - sum_e p_e R_e).
+ * R and alpha / n_l are formed in fp64 and rounded to fp32; the rest is fp32
+ * (expf, sums over the token's experts, no fused multiply-add).
+ *   grad_s     device fp32 [T,E], 16-byte aligned (in/out)
+ *   z          device bf16 [T,E], 16-byte aligned (in): the unbiased logits
+ *   loads      device int32 [M,E] (in), mb_offsets device int64 [M+1] (in):
+ *              as in lei_inject_grad
+ * Supported: E a multiple of 8, E <= 256, 0 <= T <= 2^31 - 2^24. */
+eqb_status gshard_inject_grad(float *grad_s, const eqb_bf16 *z, const int32_t *loads,
+                              const int64_t *mb_offsets, int32_t M, int64_t T, int32_t E,
+                              int32_t K, float alpha, void *stream);
+
 /* Balance metric MaxVio, Sec. 5 (Metrics) and App. E (balance metrics):
  *   MaxVio(B) = max_e [ f_e(B) / fbar(B) - 1 ],   fbar(B) = K |B| / E,
  * in fp64 (fbar formed as (K * |B|) / E, then one division and one

@@ -32,7 +32,7 @@ __all__ = [
     "eqb_margin_hist_pass2", "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad",
     "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route", "eqb_router_layer_step",
-    "eqb_maxvio",
+    "eqb_maxvio", "gshard_inject_grad",
 ]
 
 
@@ -186,6 +186,20 @@ def eqb_router_route(x, W_r, b, K, mb_offsets=None, z=None, topk_idx=None, tau=N
                                    _p(topk_idx), _p(tau), _p(loads), _p(err_flag), _stream(stream)),
            "eqb_router_route")
     return z, topk_idx, tau
+
+
+def gshard_inject_grad(grad_s, z, loads, mb_offsets, K, alpha, stream=None):
+    """GShard auxiliary-loss gradient added to grad_s in place (see eqb.h):
+    grad_s fp32 [T,E], z bf16 [T,E], loads int32 [M,E], mb_offsets int64."""
+    T, E = z.shape
+    _need(grad_s, torch.float32, "grad_s", (T, E))
+    _need(z, torch.bfloat16, "z")
+    _need(mb_offsets, torch.int64, "mb_offsets")
+    M = mb_offsets.numel() - 1
+    _need(loads, torch.int32, "loads", (M, E))
+    _check(load().gshard_inject_grad(_p(grad_s), _p(z), _p(loads), _p(mb_offsets), M, T, E, K,
+                                     float(alpha), _stream(stream)), "gshard_inject_grad")
+    return grad_s
 
 
 def eqb_maxvio(loads, mb_offsets, K, out=None, per_mb=None, stream=None):

@@ -17,7 +17,7 @@ EXPORTS = (
     "eqb_margin_hist_pass1", "eqb_margin_hist_pass2", "eqb_select_quantile",
     "eqb_bias_update", "lei_inject_grad", "eqb_router_logits", "eqb_layer_workspace_bytes",
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route",
-    "eqb_router_layer_step", "eqb_maxvio",
+    "eqb_router_layer_step", "eqb_maxvio", "gshard_inject_grad",
 )
 
 STATUS = {0: "EQB_OK", 1: "EQB_ERR_INVALID_ARG", 2: "EQB_ERR_UNSUPPORTED", 3: "EQB_ERR_CUDA",
@@ -54,6 +54,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
             "lei_inject_grad": [P, P, P, i32, i64, i32, i32, f32, f32, P],
             "eqb_router_logits": [P, P, i64, i32, i32, P, P, P],
             "eqb_maxvio": [P, P, i32, i32, i32, P, P, P],
+            "gshard_inject_grad": [P, P, P, P, i32, i64, i32, i32, f32, P],
             "eqb_router_route": [P, P, i64, i32, i32, i32, P, P, i32, P, P, P, P, P, P],
             "eqb_router_layer_step": [P, P, i64, i32, i32, i32, P, P, P, i32, i64, P, P, P, P, P, P,
                                       f32, f32, P, ctypes.c_size_t, P, P],

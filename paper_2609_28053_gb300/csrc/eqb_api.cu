@@ -193,4 +193,18 @@ eqb_status eqb_maxvio(const int32_t* loads, const int64_t* mb_offsets, int32_t M
   return to_status(eqb::launch_maxvio(loads, mb_offsets, M, E, K, maxvio, per_mb, as_stream(stream)));
 }
 
+eqb_status gshard_inject_grad(float* grad_s, const eqb_bf16* z, const int32_t* loads, const int64_t* mb_offsets,
+                              int32_t M, int64_t T, int32_t E, int32_t K, float alpha, void* stream) {
+  if (T < 0 || E < 1 || K < 1 || M < 1) return EQB_ERR_INVALID_ARG;
+  if ((E % 8) != 0 || E > 256) return EQB_ERR_UNSUPPORTED;
+  if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
+  if (!(alpha == alpha) || alpha == INFINITY || alpha == -INFINITY) return EQB_ERR_INVALID_ARG;
+  if (!grad_s || !z || !loads || !mb_offsets) return EQB_ERR_INVALID_ARG;
+  if (!aligned(grad_s, 16) || !aligned(z, 16) || !aligned(loads, 4) || !aligned(mb_offsets, 8))
+    return EQB_ERR_INVALID_ARG;
+  if (T == 0) return EQB_OK;
+  eqb::GshardArgs a{grad_s, z, loads, mb_offsets, M, T, E, K, alpha};
+  return to_status(eqb::launch_gshard(a, as_stream(stream)));
+}
+
 }  // extern "C"

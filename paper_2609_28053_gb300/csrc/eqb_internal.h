@@ -60,6 +60,17 @@ struct LeiArgs {
   float eta, c;
 };
 
+struct GshardArgs {
+  float* g;
+  const uint16_t* z;
+  const int32_t* loads;
+  const int64_t* off;
+  int M;
+  int64_t T;
+  int E, K;
+  float alpha;
+};
+
 int launch_route(const RouteArgs& a, cudaStream_t s);
 bool route_wide_supported(int E, int K);
 int launch_route_wide(const RouteArgs& a, cudaStream_t s);
@@ -70,6 +81,7 @@ int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t
 int launch_lei(const LeiArgs& a, cudaStream_t s);
 int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, uint16_t* z,
                        int32_t* err, cudaStream_t s);
+int launch_gshard(const GshardArgs& a, cudaStream_t s);
 int launch_maxvio(const int32_t* loads, const int64_t* off, int M, int E, int K, double* out, double* per_mb,
                   cudaStream_t s);
 int launch_router_route(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, int K, const float* b,

@@ -1,0 +1,131 @@
+// gshard.cu -- the GShard auxiliary-loss gradient, the comparison injection
+// beside LEI (arXiv 2609.28053, Sec. 2 and App. D, Eq. (gshard-grad)):
+//   grad_s[t, j] += alpha / (n_l d_t) * (R_j - sum_e p_{t,e} R_e),
+// with R_e = f_{l,e} / (K n_l) - 1/E for the token's microbatch l (n_l
+// tokens), s = sigmoid(z), d_t = sum_e s_{t,e} and p = s / d_t.
+//
+// A stream like LEI (z read once, grad_s read and written once).  Each CTA
+// takes a contiguous token range and, for every microbatch it meets, forms R
+// (fp64, rounded to fp32) and alpha / n_l in shared memory.  LPT lanes share
+// a token, 8 experts per lane (one 16-byte load of z, two of grad_s); the
+// score sum and the R-weighted sum are reduced over those lanes with
+// shuffles, then each lane updates its 8 gradients.
+#include "eqb_device.cuh"
+
+namespace eqb {
+
+namespace {
+
+constexpr int kGsThreads = 256;
+
+template <int LPT>
+__global__ void __launch_bounds__(kGsThreads) gshard_kernel(GshardArgs a, int64_t tokens_per_cta) {
+  constexpr int TPW = 32 / LPT;  // tokens per warp step
+  __shared__ __align__(16) float Rs[256];
+  __shared__ float cs;
+  const int E = a.E, nch = E >> 3;
+  const int64_t tb = (int64_t)blockIdx.x * tokens_per_cta;
+  const int64_t te = min(tb + tokens_per_cta, a.T);
+  if (tb >= te) return;
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  const int sub = lane & (LPT - 1), slot = lane / LPT;
+  const bool has_chunk = sub < nch;
+
+  int64_t t = tb;
+  while (t < te) {
+    const int l = microbatch_of(a.off, a.M, t);
+    const int64_t lo = __ldg(a.off + l), hi = __ldg(a.off + l + 1);
+    const int64_t seg_end = (hi > t) ? min(te, hi) : te;
+    __syncthreads();  // the previous segment is done with Rs and cs
+    const int64_t n = hi - lo;
+    if (threadIdx.x < E)
+      Rs[threadIdx.x] =
+          n > 0 ? __double2float_rn((double)__ldg(a.loads + (int64_t)l * E + threadIdx.x) / ((double)a.K * (double)n) -
+                                    1.0 / (double)E)
+                : 0.f;
+    if (threadIdx.x == 0) cs = n > 0 ? __double2float_rn((double)a.alpha / (double)n) : 0.f;
+    __syncthreads();
+    float r[8];
+    if (has_chunk) {
+      const float4 r0 = reinterpret_cast<const float4*>(Rs)[2 * sub];
+      const float4 r1 = reinterpret_cast<const float4*>(Rs)[2 * sub + 1];
+      r[0] = r0.x; r[1] = r0.y; r[2] = r0.z; r[3] = r0.w;
+      r[4] = r1.x; r[5] = r1.y; r[6] = r1.z; r[7] = r1.w;
+    } else {
+#pragma unroll
+      for (int i = 0; i < 8; ++i) r[i] = 0.f;
+    }
+    const float c0 = cs;
+
+    for (int64_t base = t + (int64_t)wid * TPW; base < seg_end; base += (int64_t)nw * TPW) {
+      const int64_t tok = base + slot;
+      const bool ok = has_chunk && tok < seg_end;
+      float s[8];
+      float d = 0.f, num = 0.f;
+      if (ok) {
+        const uint4 w = __ldcs(reinterpret_cast<const uint4*>(a.z + tok * E) + sub);
+        const uint32_t zw[4] = {w.x, w.y, w.z, w.w};
+#pragma unroll
+        for (int q = 0; q < 4; ++q) {
+          s[2 * q] = 1.0f / (1.0f + expf(-bf16_lo(zw[q])));
+          s[2 * q + 1] = 1.0f / (1.0f + expf(-bf16_hi(zw[q])));
+        }
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          d = __fadd_rn(d, s[i]);
+          num = __fadd_rn(num, __fmul_rn(s[i], r[i]));
+        }
+      }
+#pragma unroll
+      for (int m = 1; m < LPT; m <<= 1) {
+        d = __fadd_rn(d, __shfl_xor_sync(kFull, d, m));
+        num = __fadd_rn(num, __shfl_xor_sync(kFull, num, m));
+      }
+      if (ok) {
+        const float mean = __fdiv_rn(num, d);
+        const float coef = __fdiv_rn(c0, d);
+        float4* gp = reinterpret_cast<float4*>(a.g + tok * E) + 2 * sub;
+        float4 g0 = __ldcs(gp), g1 = __ldcs(gp + 1);
+        g0.x = __fadd_rn(g0.x, __fmul_rn(coef, __fsub_rn(r[0], mean)));
+        g0.y = __fadd_rn(g0.y, __fmul_rn(coef, __fsub_rn(r[1], mean)));
+        g0.z = __fadd_rn(g0.z, __fmul_rn(coef, __fsub_rn(r[2], mean)));
+        g0.w = __fadd_rn(g0.w, __fmul_rn(coef, __fsub_rn(r[3], mean)));
+        g1.x = __fadd_rn(g1.x, __fmul_rn(coef, __fsub_rn(r[4], mean)));
+        g1.y = __fadd_rn(g1.y, __fmul_rn(coef, __fsub_rn(r[5], mean)));
+        g1.z = __fadd_rn(g1.z, __fmul_rn(coef, __fsub_rn(r[6], mean)));
+        g1.w = __fadd_rn(g1.w, __fmul_rn(coef, __fsub_rn(r[7], mean)));
+        __stcs(gp, g0);
+        __stcs(gp + 1, g1);
+      }
+    }
+    t = seg_end;
+  }
+}
+
+template <int LPT>
+int launch_gs(const GshardArgs& a, cudaStream_t s) {
+  DeviceInfo di;
+  if (int rc = device_info(&di)) return rc;
+  int64_t grid = (int64_t)di.sm_count * 8;
+  const int64_t max_grid = (a.T + 255) / 256;  // at least 256 tokens per CTA
+  if (grid > max_grid) grid = max_grid;
+  if (grid < 1) grid = 1;
+  const int64_t tpc = (a.T + grid - 1) / grid;
+  gshard_kernel<LPT><<<(unsigned)grid, kGsThreads, 0, s>>>(a, tpc);
+  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+}
+
+}  // namespace
+
+int launch_gshard(const GshardArgs& a, cudaStream_t s) {
+  const int nch = a.E >> 3;
+  if (nch <= 1) return launch_gs<1>(a, s);
+  if (nch <= 2) return launch_gs<2>(a, s);
+  if (nch <= 4) return launch_gs<4>(a, s);
+  if (nch <= 8) return launch_gs<8>(a, s);
+  if (nch <= 16) return launch_gs<16>(a, s);
+  if (nch <= 32) return launch_gs<32>(a, s);
+  return kErrUnsupported;
+}
+
+}  // namespace eqb

@@ -205,3 +205,15 @@ def test_maxvio_rejects(lib):
     assert f(FAKE, FAKE, 4, 8, 2, NULL, NULL, NULL) == INVALID
     assert f(FAKE, FAKE, 4, 0, 2, FAKE, NULL, NULL) == INVALID
     assert f(FAKE, FAKE, 4, 8, 2, ctypes.c_void_p(0x10004), NULL, NULL) == INVALID  # maxvio not 8-aligned
+
+
+def test_gshard_rejects(lib):
+    f = lib.gshard_inject_grad
+    a = ctypes.c_float(0.01)
+    assert f(FAKE, FAKE, FAKE, FAKE, 2, 10, 12, 2, a, NULL) == UNSUPPORTED     # E % 8
+    assert f(FAKE, FAKE, FAKE, FAKE, 2, 10, 264, 2, a, NULL) == UNSUPPORTED    # E > 256
+    assert f(NULL, FAKE, FAKE, FAKE, 2, 10, 64, 2, a, NULL) == INVALID
+    assert f(MISALIGNED, FAKE, FAKE, FAKE, 2, 10, 64, 2, a, NULL) == INVALID
+    assert f(FAKE, FAKE, FAKE, FAKE, 2, 10, 64, 2, ctypes.c_float(float("nan")), NULL) == INVALID
+    assert f(FAKE, FAKE, FAKE, FAKE, 0, 10, 64, 2, a, NULL) == INVALID
+    assert f(FAKE, FAKE, FAKE, FAKE, 2, 0, 64, 2, a, NULL) == 0
