@@ -298,6 +298,70 @@ def gshard(g, z_bits, loads, offsets, K, alpha):
     return out
 
 
+def _f32_of_bf16(bits):
+    return (np.asarray(bits, np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def _center_f64(v):
+    """Eq. (2) centering of fp64 values: mean summed sequentially in ascending
+    expert order, b_e = fp32(v_e - mean)."""
+    acc = 0.0
+    for x in v:
+        acc += float(x)
+    mean = acc / len(v)
+    return np.array([np.float32(float(x) - mean) for x in v], np.float32)
+
+
+def rank_averaged_bias(z_bits, tau, K, shard_offsets):
+    """The rank-averaged QB estimate that Sec. 2 contrasts with the global
+    quantile: every data-parallel shard p takes its own K/E quantile of the
+    margins tau_t - z_{t,e} (the r_p-th smallest, r_p = ceil(n_p K / E)), the
+    shards' quantiles are averaged in fp64 (ascending p; an empty shard has
+    no quantile and is left out), and the average is centered as in Eq. (2).
+    Returns (b float32 [E], per-shard quantiles uint16 [P', E])."""
+    z_bits = _c(z_bits, np.uint16)
+    T, E = z_bits.shape
+    tau = _c(tau, np.float32)
+    off = np.asarray(shard_offsets, np.int64)
+    qs = []
+    for p in range(len(off) - 1):
+        a, b = int(off[p]), int(off[p + 1])
+        if b == a:
+            continue
+        qs.append(quantile(z_bits[a:b], tau[a:b], target_rank(b - a, E, K)))
+    qs = np.array(qs, np.uint16)
+    avg = np.zeros(E, np.float64)
+    for e in range(E):
+        acc = 0.0
+        for p in range(len(qs)):
+            acc += float(_f32_of_bf16(qs[p, e]))
+        avg[e] = acc / len(qs)
+    return _center_f64(avg), qs
+
+
+def fixed_hist_bias(z_bits, tau, K, lo, width, nbins=256):
+    """The fixed-resolution histogram estimate of Sec. 2 (histogram counts of
+    the margins summed over ranks): margin m falls in bin
+    j = floor(fp32(fp32(m - lo) * fp32(1 / width))) clamped to [0, nbins - 1];
+    the estimate of expert e is the upper edge lo + (j + 1) * width (fp64) of
+    the first bin whose cumulative count reaches r = ceil(T K / E), centered
+    as in Eq. (2).  Returns (b float32 [E], estimates float64 [E])."""
+    z_bits = _c(z_bits, np.uint16)
+    T, E = z_bits.shape
+    tau = _c(tau, np.float32)
+    r = target_rank(T, E, K)
+    lo32, inv_w = np.float32(lo), np.float32(np.float32(1.0) / np.float32(width))
+    est = np.zeros(E, np.float64)
+    for e in range(E):
+        m = _f32_of_bf16(margins(z_bits, tau, e))
+        x = (m - lo32) * inv_w  # float32 arithmetic, round to nearest
+        j = np.clip(np.floor(x), 0, nbins - 1).astype(np.int64)
+        counts = np.bincount(j, minlength=nbins)
+        jr = int(np.argmax(np.cumsum(counts) >= r))
+        est[e] = float(np.float32(lo)) + (jr + 1) * float(np.float32(width))
+    return _center_f64(est), est
+
+
 def eqb_step(z_bits, b, K, offsets=None):
     """The whole forward statistic of one layer on the oracle: routing, the
     exact quantile of every expert by full sort, and the centered bias."""

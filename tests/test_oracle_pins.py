@@ -459,3 +459,143 @@ def test_gshard_orthogonal_to_scores_and_zero_when_balanced():
     off_b = np.array([0, 80, 160, 200], np.int64)  # K n / E integral: n in {80, 80, 40}
     bal = np.repeat((K * np.diff(off_b) // E)[:, None], E, axis=1).astype(np.int32)
     assert np.array_equal(oracle.gshard(g, z, bal, off_b, K, 3.0), g)
+
+
+# ------------------------------------------- comparison statistics (Sec. 2)
+
+def integer_case(T, E, K, seed):
+    """Integer logits (so every score, cutoff and margin is an integer) with
+    b = 0; returns z bits and tau."""
+    rng = np.random.default_rng(seed)
+    z = brute.bf16_bits_from_f32(rng.integers(-8, 9, size=(T, E)).astype(np.float32))
+    _, tau, _ = oracle.route(z, np.zeros(E, np.float32), K)
+    return z, tau
+
+
+def pin_rank_avg_single_shard_is_eqb(fn):
+    rng = np.random.default_rng(1)
+    T, E, K = 300, 16, 2
+    z = brute.bf16_bits_from_f32(rng.standard_normal((T, E)).astype(np.float32))
+    st = oracle.eqb_step(z, np.zeros(E, np.float32), K)
+    b, _ = fn(z, st["tau"], K, [0, T])
+    assert np.array_equal(b, st["b_next"])
+
+
+def pin_rank_avg_against_sorted_shards(fn):
+    """Each shard's quantile by numpy's sort of its margins, the average and
+    the centering in exact rationals."""
+    from fractions import Fraction
+    rng = np.random.default_rng(2)
+    T, E, K = 240, 8, 3
+    z = brute.bf16_bits_from_f32(rng.standard_normal((T, E)).astype(np.float32))
+    _, tau, _ = oracle.route(z, np.zeros(E, np.float32), K)
+    off = [0, 40, 40, 130, 240]  # includes an empty shard
+    b, _ = fn(z, tau, K, off)
+    zf = brute.f32_from_bf16_bits(z)
+    avg = []
+    for e in range(E):
+        qs = []
+        for p in range(len(off) - 1):
+            a, c = off[p], off[p + 1]
+            if c == a:
+                continue
+            m = brute.f32_from_bf16_bits(brute.bf16_bits_from_f32((tau[a:c] - zf[a:c, e]).astype(np.float32)))
+            r = -(-(c - a) * K // E)
+            qs.append(Fraction(float(np.sort(m)[r - 1])))
+        avg.append(sum(qs, Fraction(0)) / len(qs))
+    mean = sum(avg, Fraction(0)) / E
+    want = np.array([float(a - mean) for a in avg])
+    assert np.all(np.abs(b.astype(np.float64) - want) <= 2.0 ** -20 * np.maximum(1.0, np.abs(want)))
+
+
+def pin_fixed_hist_integer_grid_is_eqb(fn):
+    """Integer margins and unit bins centred on the integers: every margin has
+    its own bin, the estimate is the r-th smallest margin + 1/2, and the shift
+    cancels in the centering (E a power of two keeps the mean exact)."""
+    T, E, K = 400, 16, 2
+    z, tau = integer_case(T, E, K, seed=3)
+    st = oracle.eqb_step(z, np.zeros(E, np.float32), K)
+    b, est = fn(z, tau, K, -64.5, 1.0)
+    assert np.array_equal(est, brute.f32_from_bf16_bits(st["qhat"]).astype(np.float64) + 0.5)
+    assert np.array_equal(b, st["b_next"])
+
+
+def pin_fixed_hist_is_bin_of_rth_margin(fn):
+    """The first bin whose cumulative count reaches r is the bin that holds
+    the r-th smallest margin (order statistic from numpy's sort)."""
+    rng = np.random.default_rng(4)
+    T, E, K = 300, 8, 2
+    z = brute.bf16_bits_from_f32(rng.standard_normal((T, E)).astype(np.float32))
+    _, tau, _ = oracle.route(z, np.zeros(E, np.float32), K)
+    lo, w = -2.0, 0.0625
+    _, est = fn(z, tau, K, lo, w, nbins=64)
+    zf = brute.f32_from_bf16_bits(z)
+    r = -(-T * K // E)
+    inv = np.float32(np.float32(1.0) / np.float32(w))
+    for e in range(E):
+        m = np.sort(brute.f32_from_bf16_bits(brute.bf16_bits_from_f32((tau - zf[:, e]).astype(np.float32))))[r - 1]
+        j = int(min(max(np.floor((np.float32(m) - np.float32(lo)) * inv), 0), 63))
+        assert est[e] == lo + (j + 1) * w
+
+
+COMPARISON_PINS = {
+    "rank_avg": [pin_rank_avg_single_shard_is_eqb, pin_rank_avg_against_sorted_shards],
+    "fixed_hist": [pin_fixed_hist_integer_grid_is_eqb, pin_fixed_hist_is_bin_of_rth_margin],
+}
+
+
+@pytest.mark.parametrize("pin", COMPARISON_PINS["rank_avg"], ids=lambda f: f.__name__)
+def test_rank_averaged_bias_pins(pin):
+    pin(oracle.rank_averaged_bias)
+
+
+@pytest.mark.parametrize("pin", COMPARISON_PINS["fixed_hist"], ids=lambda f: f.__name__)
+def test_fixed_hist_bias_pins(pin):
+    pin(oracle.fixed_hist_bias)
+
+
+def _rank_avg_size_weighted(z_bits, tau, K, off):
+    """A plausible mistake: shards weighted by their token counts."""
+    T, E = z_bits.shape
+    num = np.zeros(E)
+    for p in range(len(off) - 1):
+        a, c = off[p], off[p + 1]
+        if c > a:
+            q = oracle.quantile(z_bits[a:c], tau[a:c], oracle.target_rank(c - a, E, K))
+            num += (c - a) * brute.f32_from_bf16_bits(q)
+    avg = num / T
+    return (avg - avg.mean()).astype(np.float32), None
+
+
+def _rank_avg_global_rank(z_bits, tau, K, off):
+    """A plausible mistake: every shard uses the global rank r = ceil(TK/E)."""
+    T, E = z_bits.shape
+    qs = []
+    for p in range(len(off) - 1):
+        a, c = off[p], off[p + 1]
+        if c > a:
+            qs.append(brute.f32_from_bf16_bits(oracle.quantile(z_bits[a:c], tau[a:c],
+                                                               min(c - a, oracle.target_rank(T, E, K)))))
+    avg = np.mean(qs, axis=0).astype(np.float64)
+    return (avg - avg.mean()).astype(np.float32), None
+
+
+def _fixed_hist_lower_edge(z_bits, tau, K, lo, w, nbins=256):
+    """A plausible mistake: the lower bin edge as the estimate."""
+    b, est = oracle.fixed_hist_bias(z_bits, tau, K, lo, w, nbins)
+    est = est - w
+    return (est - est.mean()).astype(np.float32), est
+
+
+@pytest.mark.parametrize("kind,wrong", [("rank_avg", _rank_avg_size_weighted),
+                                        ("rank_avg", _rank_avg_global_rank),
+                                        ("fixed_hist", _fixed_hist_lower_edge)],
+                         ids=["size_weighted", "global_rank", "lower_edge"])
+def test_comparison_pins_reject_planted_mistakes(kind, wrong):
+    failed = 0
+    for pin in COMPARISON_PINS[kind]:
+        try:
+            pin(wrong)
+        except AssertionError:
+            failed += 1
+    assert failed > 0
