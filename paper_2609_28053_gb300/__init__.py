@@ -32,7 +32,7 @@ __all__ = [
     "eqb_margin_hist_pass2", "eqb_select_quantile", "eqb_bias_update", "lei_inject_grad",
     "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route", "eqb_router_layer_step",
-    "eqb_maxvio", "gshard_inject_grad",
+    "eqb_maxvio", "gshard_inject_grad", "eqb_rank_averaged_bias", "eqb_fixed_hist_bias",
 ]
 
 
@@ -200,6 +200,52 @@ def gshard_inject_grad(grad_s, z, loads, mb_offsets, K, alpha, stream=None):
     _check(load().gshard_inject_grad(_p(grad_s), _p(z), _p(loads), _p(mb_offsets), M, T, E, K,
                                      float(alpha), _stream(stream)), "gshard_inject_grad")
     return grad_s
+
+
+def eqb_rank_averaged_bias(z, tau, K, shard_offsets_host, workspace, b_out=None, q_shards=None,
+                           err_flag=None, stream=None):
+    """Rank-averaged QB (Sec. 2): each shard's own K/E margin quantile,
+    averaged over the non-empty shards and centered.  shard_offsets_host: int64
+    host array [P+1].  Returns (b fp32 [E], q_shards bf16 [P,E])."""
+    import numpy as np
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(tau, torch.float32, "tau", (T,))
+    off = np.ascontiguousarray(np.asarray(shard_offsets_host), dtype=np.int64)
+    P = len(off) - 1
+    if b_out is None:
+        b_out = torch.empty(E, dtype=torch.float32, device=z.device)
+    if q_shards is None:
+        q_shards = torch.zeros((P, E), dtype=torch.bfloat16, device=z.device)
+    _need(b_out, torch.float32, "b_out", (E,))
+    _need(q_shards, torch.bfloat16, "q_shards", (P, E))
+    _need(workspace, torch.uint8, "workspace")
+    _need(err_flag, torch.int32, "err_flag")
+    _check(load().eqb_rank_averaged_bias(_p(z), _p(tau), T, E, K, off.ctypes.data_as(ctypes.c_void_p), P,
+                                         _p(q_shards), _p(b_out), _p(workspace), workspace.numel(),
+                                         _p(err_flag), _stream(stream)), "eqb_rank_averaged_bias")
+    return b_out, q_shards
+
+
+def eqb_fixed_hist_bias(z, tau, K, lo, width, workspace, b_out=None, estimate=None, err_flag=None,
+                        stream=None):
+    """Fixed-resolution (256 equal bins) histogram estimate of the K/E margin
+    quantile (Sec. 2), centered.  Returns (b fp32 [E], estimate fp64 [E])."""
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(tau, torch.float32, "tau", (T,))
+    if b_out is None:
+        b_out = torch.empty(E, dtype=torch.float32, device=z.device)
+    if estimate is None:
+        estimate = torch.empty(E, dtype=torch.float64, device=z.device)
+    _need(b_out, torch.float32, "b_out", (E,))
+    _need(estimate, torch.float64, "estimate", (E,))
+    _need(workspace, torch.uint8, "workspace")
+    _need(err_flag, torch.int32, "err_flag")
+    _check(load().eqb_fixed_hist_bias(_p(z), _p(tau), T, E, K, float(lo), float(width), _p(b_out),
+                                      _p(estimate), _p(workspace), workspace.numel(), _p(err_flag),
+                                      _stream(stream)), "eqb_fixed_hist_bias")
+    return b_out, estimate
 
 
 def eqb_maxvio(loads, mb_offsets, K, out=None, per_mb=None, stream=None):

@@ -47,6 +47,7 @@ struct HistArgs {
   const uint8_t* u;  // pass 2 only
   int32_t* hist;
   int32_t* err;
+  float lo = 0.f, inv_w = 0.f;  // pass 3 (equal-width bins) only
 };
 
 struct LeiArgs {
@@ -70,6 +71,18 @@ struct GshardArgs {
   int E, K;
   float alpha;
 };
+
+// The step's scratch, carved from one caller-provided buffer (256-byte
+// aligned pieces): the two [E,256] histograms, u, rho and q_hat.
+struct StepWorkspace {
+  int32_t* H;
+  int32_t* L;
+  uint8_t* u;
+  int32_t* rho;
+  uint16_t* q;
+};
+// Carves `base` (or, with base == nullptr, only measures); returns the bytes used.
+size_t carve_workspace(void* base, int E, StepWorkspace* w);
 
 int launch_route(const RouteArgs& a, cudaStream_t s);
 bool route_wide_supported(int E, int K);

@@ -6,6 +6,8 @@
 // pass rescans the local margins).  Keys are kappa(m) (negative patterns
 // complemented, others with the sign bit set).  Pass 1 counts the high byte of
 // every key; pass 2 counts the low byte of the keys whose high byte is u_e.
+// Pass 3 is the fixed-resolution histogram that Sec. 2 compares against:
+// 256 equal bins, j = floor((m - lo) * inv_w) clamped to [0, 255].
 //
 // Work per element is kept to a handful of instructions by working on packed
 // pairs: one 32-bit word of z holds two experts, their two fp32 differences
@@ -88,6 +90,13 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
         const bool same = he == ho;
         red_shared_add(row + 4u * he, same ? 0x10001u : 1u);
         if (!same) red_shared_add(row + 4u * ho, 0x10000u);
+      } else if (PASS == 3) {
+        // equal-width bins: j = floor((m - lo) * inv_w), clamped to [0, 255]
+        const uint32_t he = static_cast<uint32_t>(min(max(__float2int_rd(__fmul_rn(__fsub_rn(bf16_lo(m), a.lo), a.inv_w)), 0), 255));
+        const uint32_t ho = static_cast<uint32_t>(min(max(__float2int_rd(__fmul_rn(__fsub_rn(bf16_hi(m), a.lo), a.inv_w)), 0), 255));
+        const bool same = he == ho;
+        red_shared_add(row + 4u * he, same ? 0x10001u : 1u);
+        if (!same) red_shared_add(row + 4u * ho, 0x10000u);
       } else {
         const uint32_t d = (k ^ sel[p]) & 0xff00ff00u;
         if ((d & 0x0000ff00u) == 0u) red_shared_add(row + 4u * (k & 0xffu), 1u);
@@ -125,7 +134,7 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
       const uint32_t v = bins[wi];
       if (v) {
         bins[wi] = 0u;
-        const int bin = (PASS == 1) ? (slot ^ 0x80) : slot;
+        const int bin = (PASS == 1) ? (slot ^ 0x80) : slot;  // pass 1 stores internal keys
         const int ee = e0 + 2 * row;
         if (v & 0xffffu) atomicAdd(a.hist + (int64_t)ee * 256 + bin, static_cast<int>(v & 0xffffu));
         if (v >> 16) atomicAdd(a.hist + (int64_t)(ee + 1) * 256 + bin, static_cast<int>(v >> 16));
@@ -173,6 +182,7 @@ int launch_hist_pass(const HistArgs& a, cudaStream_t s) {
 }  // namespace
 
 int launch_hist(const HistArgs& a, int pass, cudaStream_t s) {
+  if (pass == 3) return launch_hist_pass<3>(a, s);
   return pass == 1 ? launch_hist_pass<1>(a, s) : launch_hist_pass<2>(a, s);
 }
 

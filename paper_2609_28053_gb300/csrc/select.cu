@@ -7,6 +7,10 @@
 //   pass 1: u_e = min{u : sum_{j<=u} H[e][j] >= r},  rho_e = r - sum_{j<u_e} H[e][j]
 //   pass 2: v_e = min{v : sum_{j<=v} L[e][j] >= rho_e},
 //           q_hat_e = kappa^{-1}((u_e << 8) | v_e)   (a zero returned as +0)
+//   pass 3: pass 1 on a histogram of equal-width bins, whose edge bins hold
+//           ordinary (clamped) margins rather than non-finite ones
+//   pass 3: as pass 1 on a histogram of equal-width bins, where the edge bins
+//           hold ordinary (clamped) values rather than non-finite margins
 // The bias update reproduces the definition's fp64 sum in ascending expert
 // order bit for bit (see bias_update_kernel), divides by E and subtracts.
 #include "eqb_device.cuh"
@@ -37,14 +41,15 @@ __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__
     if (lane >= d) incl += o;
   }
   const int64_t excl = incl - local;
-  const int64_t target = (pass == 1) ? r : (int64_t)rho[e];
+  const bool first = pass != 2;
+  const int64_t target = first ? r : (int64_t)rho[e];
   const unsigned hit = __ballot_sync(kFull, excl < target && target <= incl);
   if (pass == 1 && ((lane == 0 && cnt[0] != 0) || (lane == 31 && cnt[7] != 0)))
     raise_flag(err, kErrNonfinite);
   if (hit == 0u || target < 1) {
     if (lane == 0) {
       raise_flag(err, kErrRank);
-      if (pass == 1) { u[e] = 255; rho[e] = 0; }
+      if (first) { u[e] = 255; rho[e] = 0; }
       else q_hat[e] = 0x7fc0;  // NaN marks an unreachable rank
     }
     return;
@@ -55,7 +60,7 @@ __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__
     for (int j = 0; j < 8; ++j) {
       if (below + cnt[j] >= target) {
         const int bin = lane * 8 + j;
-        if (pass == 1) {
+        if (first) {
           u[e] = static_cast<uint8_t>(bin);
           rho[e] = static_cast<int32_t>(target - below);
         } else {

@@ -12,24 +12,13 @@
 #include "eqb.h"
 #include "eqb_internal.h"
 
-namespace {
+namespace eqb {
 
-size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
-
-struct Workspace {
-  int32_t* H;
-  int32_t* L;
-  uint8_t* u;
-  int32_t* rho;
-  uint16_t* q;
-};
-
-// Carve the caller's workspace (or, with base == NULL, only measure it).
-size_t carve(void* base, int E, Workspace* w) {
+size_t carve_workspace(void* base, int E, StepWorkspace* w) {
   size_t off = 0;
   auto take = [&](size_t n) {
     uint8_t* p = base ? static_cast<uint8_t*>(base) + off : nullptr;
-    off = align_up(off + n, 256);
+    off = (off + n + 255) / 256 * 256;
     return p;
   };
   w->H = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 256 * 4));
@@ -39,6 +28,13 @@ size_t carve(void* base, int E, Workspace* w) {
   w->q = reinterpret_cast<uint16_t*>(take(static_cast<size_t>(E) * 2));
   return off;
 }
+
+}  // namespace eqb
+
+namespace {
+
+using Workspace = eqb::StepWorkspace;
+inline size_t carve(void* base, int E, Workspace* w) { return eqb::carve_workspace(base, E, w); }
 
 inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 inline eqb_status st(int rc) { return static_cast<eqb_status>(rc); }

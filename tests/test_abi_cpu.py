@@ -217,3 +217,27 @@ def test_gshard_rejects(lib):
     assert f(FAKE, FAKE, FAKE, FAKE, 2, 10, 64, 2, ctypes.c_float(float("nan")), NULL) == INVALID
     assert f(FAKE, FAKE, FAKE, FAKE, 0, 10, 64, 2, a, NULL) == INVALID
     assert f(FAKE, FAKE, FAKE, FAKE, 2, 0, 64, 2, a, NULL) == 0
+
+
+def test_comparison_statistics_reject(lib):
+    import numpy as np
+    ws = lib.eqb_layer_workspace_bytes(64)
+    good = np.array([0, 40, 100], np.int64)
+    bad = np.array([0, 60, 50], np.int64)
+    f = lib.eqb_rank_averaged_bias
+
+    def ra(off=good, P=2, q=FAKE, wsb=ws, E=64):
+        return f(FAKE, FAKE, 100, E, 8, None if off is None else off.ctypes.data_as(ctypes.c_void_p), P, q,
+                 FAKE, FAKE, wsb, NULL, NULL)
+    assert ra(off=bad) == INVALID
+    assert ra(off=None) == INVALID
+    assert ra(q=NULL) == INVALID
+    assert ra(wsb=ws - 1) == INVALID
+    assert ra(E=72 + 200) == UNSUPPORTED
+    g = lib.eqb_fixed_hist_bias
+    fl = ctypes.c_float
+    assert g(FAKE, FAKE, 100, 64, 8, fl(-1.0), fl(0.0), FAKE, NULL, FAKE, ws, NULL, NULL) == INVALID
+    assert g(FAKE, FAKE, 100, 64, 8, fl(float("nan")), fl(0.1), FAKE, NULL, FAKE, ws, NULL, NULL) == INVALID
+    assert g(FAKE, FAKE, 100, 64, 8, fl(-1.0), fl(0.1), FAKE, NULL, FAKE, ws - 1, NULL, NULL) == INVALID
+    assert g(FAKE, FAKE, 100, 64, 8, fl(-1.0), fl(0.1), FAKE, ctypes.c_void_p(0x10004), FAKE, ws, NULL,
+             NULL) == INVALID
