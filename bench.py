@@ -280,21 +280,23 @@ def run_reference(args):
     ws, rank, local = dist_env()
     if rank != 0:
         return
-    sh = SHAPES["global"]
+    wl = args.workload if args.workload != "router" else "global"
+    sh = SHAPES[wl]
     n = args.ref_sample_tokens
-    z = make_logits("global", T=n, device="cpu")
-    b = make_bias("global", device="cpu")
-    g = make_grad("global", T=n, device="cpu")
+    per = sh.T // sh.M
+    z = make_logits(wl, T=n, device="cpu")
+    b = make_bias(wl, device="cpu")
+    g = make_grad(wl, T=n, device="cpu")
     for _ in range(args.warmup):
-        cpu_oracle_sample(z, b, g, sh.K, n, 32768)
-    times = [cpu_oracle_sample(z, b, g, sh.K, n, 32768)[0] for _ in range(args.steps)]
+        cpu_oracle_sample(z, b, g, sh.K, n, per)
+    times = [cpu_oracle_sample(z, b, g, sh.K, n, per)[0] for _ in range(args.steps)]
     tot = sum(times)
     value = args.steps * n / tot
     line = {"impl": "reference", "metric": METRIC, "value": value, "unit": "tokens/s",
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": 1e3 * tot / args.steps, "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f32", "data": "synthetic",
-            "config": {"workload": f"global: T={sh.T} E={sh.E} K={sh.K} M={sh.M}, oracle on a "
+            "config": {"workload": f"{wl}: T={sh.T} E={sh.E} K={sh.K} M={sh.M}, oracle on a "
                                    f"{n}-token sample per step", "T": sh.T, "E": sh.E, "K": sh.K},
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                              "sample": f"first {n} tokens of the workload per step",
@@ -304,18 +306,86 @@ def run_reference(args):
     print(json.dumps(line), flush=True)
 
 
+def time_call(fn, stream, reps=10):
+    """Mean CUDA-event duration (ms) of fn() on `stream`, after one warm-up."""
+    fn()
+    torch.cuda.synchronize()
+    a, b = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    a.record(stream)
+    for _ in range(reps):
+        fn()
+    b.record(stream)
+    torch.cuda.synchronize()
+    return a.elapsed_time(b) / reps
+
+
+def extras(step, stream, peak):
+    """The comparison rows, timed beside the step (not part of it): the GShard
+    gradient (the injection LEI is compared with), MaxVio, the rank-averaged
+    and the fixed-resolution estimates of Sec. 2; and the balance each bias
+    gives on a fresh batch of the same distribution (Global and Local MaxVio
+    after one update)."""
+    eqb = step.eqb
+    T, E, K, M = step.T, step.E, step.K, step.M
+    z, off, dev = step.z, step.off, step.z.device
+    shards = even_offsets(T, M)
+    lo, width = -4.0, 1.0 / 32
+    out = {}
+
+    def row(name, ms, nbytes):
+        gbs = nbytes / (ms * 1e-3) / 1e9
+        out[name] = {"ms": round(ms, 5), "algorithmic_bytes": nbytes, "GB/s": round(gbs, 1),
+                     "frac": round(gbs / peak, 4)}
+
+    g2 = step.g.clone()
+    row("gshard_inject_grad", time_call(lambda: eqb.gshard_inject_grad(g2, z, step.loads, off, K, 1e-2, stream),
+                                        stream), 10 * T * E)
+    del g2
+    mv = torch.empty(2, dtype=torch.float64, device=dev)
+    out["maxvio"] = {"ms": round(time_call(lambda: eqb.eqb_maxvio(step.loads, off, K, out=mv, stream=stream),
+                                           stream), 5)}
+    row("rank_averaged_bias", time_call(lambda: eqb.eqb_rank_averaged_bias(
+        z, step.tau, K, shards, step.workspace, stream=stream), stream, reps=3), 2 * (2 * T * E + 4 * T))
+    row("fixed_hist_bias", time_call(lambda: eqb.eqb_fixed_hist_bias(
+        z, step.tau, K, lo, width, step.workspace, stream=stream), stream), 2 * T * E + 4 * T)
+
+    # Balance after one update: each bias routes a fresh batch.
+    b0 = step.b.clone()
+    loads = torch.zeros_like(step.loads)
+    tau = torch.empty_like(step.tau)
+    eqb.eqb_layer_step(z, b0, K, off, loads, step.b_next, step.workspace, tau=tau, mb_offsets_host=step.off_h,
+                       stream=stream)
+    biases = {"before": b0, "eqb": step.b_next.clone(),
+              "rank_averaged": eqb.eqb_rank_averaged_bias(z, tau, K, shards, step.workspace, stream=stream)[0].clone(),
+              "fixed_hist": eqb.eqb_fixed_hist_bias(z, tau, K, lo, width, step.workspace, stream=stream)[0].clone()}
+    fresh = make_logits(step.workload, T=T, seed=SHAPES[step.workload].seed + 977, device=str(dev))
+    bal = {}
+    for name, bb in biases.items():
+        loads.zero_()
+        eqb.eqb_route_topk(fresh, bb, K, off, None, tau, loads, None, None, stream)
+        eqb.eqb_maxvio(loads, off, K, out=mv, stream=stream)
+        g_, l_ = mv.tolist()
+        bal[name] = {"maxvio_global": round(g_, 4), "maxvio_local": round(l_, 4)}
+    out["maxvio_after_one_update"] = {
+        "batch": f"fresh {step.workload} batch, seed +977; biases from the timed batch",
+        "rank_averaged_shards": M, "fixed_hist_bins": f"256 x {width} from {lo}", **bal}
+    del fresh
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="global", choices=["global", "router"])
+    ap.add_argument("--workload", default="global", choices=["global", "router", "paper"])
     ap.add_argument("--tokens", type=int, default=None)
     ap.add_argument("--e2e-steps", type=int, default=3)
     ap.add_argument("--cpu-sample-tokens", type=int, default=131072)
     ap.add_argument("--ref-sample-tokens", type=int, default=32768)
     ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-extras", action="store_true")
     ap.add_argument("--traffic-file", default=os.path.join(ROOT, "profiles", "dram_traffic_per_launch.txt"))
     args = ap.parse_args()
     if args.warmup < 3 and args.impl == "ours":
@@ -442,28 +512,33 @@ def main():
 
     cpu_base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        n = min(args.cpu_sample_tokens if args.workload == "global" else 8192, T)
+        n = min(args.cpu_sample_tokens if args.workload != "router" else 8192, T)
         if args.workload == "router":
             secs, toks = cpu_oracle_router_sample(step.x, step.W, step.g, K, n)
             what = (f"first {n} tokens: router projection in fp64, routing, exact quantile of all "
                     f"{E} experts by full sort, bias update, LEI")
         else:
-            secs, toks = cpu_oracle_sample(step.z, step.b, step.g, K, n, 32768)
-            what = (f"first {n} tokens of the workload ({max(1, n // 32768)} microbatches): routing, "
+            per = T // M
+            secs, toks = cpu_oracle_sample(step.z, step.b, step.g, K, n, per)
+            what = (f"first {n} tokens of the workload ({max(1, n // per)} microbatches): routing, "
                     f"exact quantile of all {E} experts by full sort, bias update, LEI")
         cpu_base = {"value": toks / secs, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                     "sample": what, "seconds": secs,
                     "host_cores_available": len(os.sched_getaffinity(0))}
+
+    ext = None
+    if rank == 0 and world == 1 and not args.no_extras and args.workload != "router":
+        ext = extras(step, stream, peak)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
                 "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms_per_step,
                 "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
                 "data": "synthetic",
-                "config": {"workload": (f"global: T={T} E={E} K={K} M={M} per GPU, bf16 logits"
-                                        if args.workload == "global" else
-                                        f"router: x [{T},{step.d}] bf16, W_r [{E},{step.d}], "
-                                        f"E={E} K={K} M={M} per GPU, bias iterated"),
+                "config": {"workload": (f"router: x [{T},{step.d}] bf16, W_r [{E},{step.d}], "
+                                        f"E={E} K={K} M={M} per GPU, bias iterated"
+                                        if args.workload == "router" else
+                                        f"{args.workload}: T={T} E={E} K={K} M={M} per GPU, bf16 logits"),
                            "T": T, "E": E, "K": K, "M": M, "eta": ETA, "c": C_NORM,
                            "l2": "inputs larger than L2 (at least 1 GiB each); no flush",
                            "parallelism": f"dp{world}"},
@@ -475,7 +550,7 @@ def main():
                 "kernels": kernels,
                 "kernels_sequential_ms": seq_ms,
                 "clocks": clk, "e2e": e2e, "cpu_baseline": cpu_base,
-                "elements_per_s": value * E}
+                "elements_per_s": value * E, "extras": ext}
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()

@@ -176,6 +176,28 @@ def test_global_config_full_size_sampled():
 
 
 @pytest.mark.slow
+def test_paper_config_full_size_sampled():
+    """The paper's own shape (Sec. 5 / App. E.1: E = 256, K = 6, 147,456 tokens
+    on each of 64 ranks, T = 9,437,184): every token's top-K and cutoff, all
+    loads, and the exact quantile of 8 sampled experts against the oracle."""
+    name = "paper"
+    sh = SHAPES[name]
+    z = bits(make_logits(name, device="cuda"))
+    b = make_bias(name, device="cuda").cpu().numpy()
+    off = even_offsets(sh.T, sh.M)
+    g = gpu_forward(z, b, sh.K, off)
+    experts = np.random.default_rng(2).choice(sh.E, 8, replace=False)
+    o = oracle_forward(z, b, sh.K, off, experts=experts)
+    assert o["r"] == 221184
+    assert np.array_equal(g["idx"], o["idx"])
+    assert np.array_equal(bits_f32(g["tau"]), bits_f32(o["tau"]))
+    assert np.array_equal(g["loads"], o["loads"])
+    assert np.array_equal(g["q"][experts], o["q"])
+    assert np.all(g["H"].sum(1) == sh.T)
+    assert g["err"][0] == 0
+
+
+@pytest.mark.slow
 def test_router_config_three_steps_on_torch_logits():
     """Router config: z = bf16(x W_r^T) (here from torch's matmul), bias
     iterated for 3 steps from b^(0) = 0 with fresh activations; each step's
