@@ -33,7 +33,7 @@
  *    offsets[M] = T, non-decreasing (empty microbatches are allowed).
  *    The library reads them on the device; they are not checked on the host.
  *  - Supported sizes: 1 <= K, K + 1 <= 32, K < E, E a multiple of 8 with
- *    E <= 256, T <= 2^31 - 2^24.  T = 0 is a valid no-op for the streaming
+ *    E <= 1024, T <= 2^31 - 2^24.  T = 0 is a valid no-op for the streaming
  *    calls.
  *  - Device buffers of bf16 logits must be 16-byte aligned; fp32 gradient
  *    buffers 16-byte aligned.  Misaligned pointers give EQB_ERR_INVALID_ARG.
@@ -233,7 +233,7 @@ eqb_status eqb_router_logits(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t T, 
  *   z          device bf16 [T,E], 16-byte aligned (in): the unbiased logits
  *   loads      device int32 [M,E] (in), mb_offsets device int64 [M+1] (in):
  *              as in lei_inject_grad
- * Supported: E a multiple of 8, E <= 256, 0 <= T <= 2^31 - 2^24. */
+ * Supported: E a multiple of 8, E <= 1024, 0 <= T <= 2^31 - 2^24. */
 eqb_status gshard_inject_grad(float *grad_s, const eqb_bf16 *z, const int32_t *loads,
                               const int64_t *mb_offsets, int32_t M, int64_t T, int32_t E,
                               int32_t K, float alpha, void *stream);
@@ -243,7 +243,7 @@ eqb_status gshard_inject_grad(float *grad_s, const eqb_bf16 *z, const int32_t *l
  * eqb_margin_hist_pass1 (so tau comes from eqb_route_topk), end with the
  * Eq. (2) centering b_e = fp32(x_e - mean(x)) (fp64, mean summed in ascending
  * expert order), and use a workspace of eqb_layer_workspace_bytes(E) bytes
- * (256-byte aligned).  Supported: E a multiple of 8, E <= 256, T >= 1.
+ * (256-byte aligned).  Supported: E a multiple of 8, E <= 1024, T >= 1.
  *
  * Rank-averaged QB: every shard p (token range [offsets[p], offsets[p+1]))
  * selects its own K/E quantile exactly (the r_p-th smallest margin,

@@ -36,7 +36,7 @@ __device__ void center_store(double* x, int E, float* b) {
 // Average of the P shard quantiles (bf16 [P,E]) per expert, summed over the
 // shards in ascending order, then centered.
 __global__ void __launch_bounds__(256) shard_average_kernel(const uint16_t* q, int P, int E, float* b) {
-  __shared__ double x[256];
+  __shared__ double x[kMaxE];
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
     double acc = 0.0;
     for (int p = 0; p < P; ++p) acc += (double)bf16_bits_to_f32(q[(int64_t)p * E + e]);
@@ -48,7 +48,7 @@ __global__ void __launch_bounds__(256) shard_average_kernel(const uint16_t* q, i
 // Upper edge lo + (u_e + 1) w of the selected bin, then centered.
 __global__ void __launch_bounds__(256) bin_edge_kernel(const uint8_t* u, int E, float lo, float w, float* b,
                                                        double* est) {
-  __shared__ double x[256];
+  __shared__ double x[kMaxE];
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
     x[e] = (double)lo + (double)(u[e] + 1) * (double)w;
     if (est) est[e] = x[e];
@@ -62,7 +62,7 @@ inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintp
 eqb_status check_common(const eqb_bf16* z, const float* tau, int64_t T, int32_t E, int32_t K, float* b_out,
                         void* workspace, int32_t* err_flag) {
   if (T < 1 || E < 2 || K < 1 || K >= E) return EQB_ERR_INVALID_ARG;
-  if (E > 256 || (E % 8) != 0) return EQB_ERR_UNSUPPORTED;
+  if (E > kMaxE || (E % 8) != 0) return EQB_ERR_UNSUPPORTED;
   if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
   if (!z || !tau || !b_out || !workspace) return EQB_ERR_INVALID_ARG;
   if (!aligned(z, 16) || !aligned(tau, 4) || !aligned(b_out, 4) || !aligned(workspace, 256) ||

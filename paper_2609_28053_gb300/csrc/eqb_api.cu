@@ -47,7 +47,7 @@ inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintp
 inline eqb_status check_shape(int64_t T, int32_t E, int32_t K, bool need_k) {
   if (T < 0 || E < 2) return EQB_ERR_INVALID_ARG;
   if (need_k && (K < 1 || K >= E)) return EQB_ERR_INVALID_ARG;
-  if (E > 256 || (E % 8) != 0) return EQB_ERR_UNSUPPORTED;
+  if (E > eqb::kMaxE || (E % 8) != 0) return EQB_ERR_UNSUPPORTED;
   if (need_k && K + 1 > 32) return EQB_ERR_UNSUPPORTED;
   // 32-bit token loop indices need headroom above T.
   if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
@@ -138,7 +138,7 @@ eqb_status eqb_select_quantile(const int32_t* hist, int32_t E, int32_t pass, int
 
 eqb_status eqb_bias_update(const eqb_bf16* q_hat, int32_t E, float* b_next, void* stream) {
   if (E < 1) return EQB_ERR_INVALID_ARG;
-  if (E > 256) return EQB_ERR_UNSUPPORTED;
+  if (E > eqb::kMaxE) return EQB_ERR_UNSUPPORTED;
   if (!q_hat || !b_next || !aligned(q_hat, 2) || !aligned(b_next, 4)) return EQB_ERR_INVALID_ARG;
   return to_status(eqb::launch_bias_update(q_hat, E, b_next, as_stream(stream)));
 }
@@ -196,7 +196,7 @@ eqb_status eqb_maxvio(const int32_t* loads, const int64_t* mb_offsets, int32_t M
 eqb_status gshard_inject_grad(float* grad_s, const eqb_bf16* z, const int32_t* loads, const int64_t* mb_offsets,
                               int32_t M, int64_t T, int32_t E, int32_t K, float alpha, void* stream) {
   if (T < 0 || E < 1 || K < 1 || M < 1) return EQB_ERR_INVALID_ARG;
-  if ((E % 8) != 0 || E > 256) return EQB_ERR_UNSUPPORTED;
+  if ((E % 8) != 0 || E > eqb::kMaxE) return EQB_ERR_UNSUPPORTED;
   if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
   if (!(alpha == alpha) || alpha == INFINITY || alpha == -INFINITY) return EQB_ERR_INVALID_ARG;
   if (!grad_s || !z || !loads || !mb_offsets) return EQB_ERR_INVALID_ARG;

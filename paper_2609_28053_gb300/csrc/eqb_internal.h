@@ -39,6 +39,10 @@ struct RouteArgs {
   int32_t* err;
 };
 
+// Largest expert count of the routing, EQB, LEI, GShard and MaxVio paths
+// (per-expert state of the per-microbatch kernels lives in shared memory).
+constexpr int kMaxE = 1024;
+
 struct HistArgs {
   const uint16_t* z;
   const float* tau;

@@ -7,9 +7,10 @@
 // A stream like LEI (z read once, grad_s read and written once).  Each CTA
 // takes a contiguous token range and, for every microbatch it meets, forms R
 // (fp64, rounded to fp32) and alpha / n_l in shared memory.  LPT lanes share
-// a token, 8 experts per lane (one 16-byte load of z, two of grad_s); the
-// score sum and the R-weighted sum are reduced over those lanes with
-// shuffles, then each lane updates its 8 gradients.
+// a token, 8 experts per lane and chunk (one 16-byte load of z, two of
+// grad_s; CPL chunks per lane when E > 256); the score sum and the
+// R-weighted sum are reduced over those lanes with shuffles, then each lane
+// updates its gradients.
 #include "eqb_device.cuh"
 
 namespace eqb {
@@ -18,10 +19,10 @@ namespace {
 
 constexpr int kGsThreads = 256;
 
-template <int LPT>
+template <int LPT, int CPL>
 __global__ void __launch_bounds__(kGsThreads) gshard_kernel(GshardArgs a, int64_t tokens_per_cta) {
   constexpr int TPW = 32 / LPT;  // tokens per warp step
-  __shared__ __align__(16) float Rs[256];
+  __shared__ __align__(16) float Rs[kMaxE];
   __shared__ float cs;
   const int E = a.E, nch = E >> 3;
   const int64_t tb = (int64_t)blockIdx.x * tokens_per_cta;
@@ -29,7 +30,6 @@ __global__ void __launch_bounds__(kGsThreads) gshard_kernel(GshardArgs a, int64_
   if (tb >= te) return;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
   const int sub = lane & (LPT - 1), slot = lane / LPT;
-  const bool has_chunk = sub < nch;
 
   int64_t t = tb;
   while (t < te) {
@@ -38,42 +38,48 @@ __global__ void __launch_bounds__(kGsThreads) gshard_kernel(GshardArgs a, int64_
     const int64_t seg_end = (hi > t) ? min(te, hi) : te;
     __syncthreads();  // the previous segment is done with Rs and cs
     const int64_t n = hi - lo;
-    if (threadIdx.x < E)
-      Rs[threadIdx.x] =
-          n > 0 ? __double2float_rn((double)__ldg(a.loads + (int64_t)l * E + threadIdx.x) / ((double)a.K * (double)n) -
-                                    1.0 / (double)E)
-                : 0.f;
+    for (int e = threadIdx.x; e < E; e += blockDim.x)
+      Rs[e] = n > 0 ? __double2float_rn((double)__ldg(a.loads + (int64_t)l * E + e) / ((double)a.K * (double)n) -
+                                        1.0 / (double)E)
+                    : 0.f;
     if (threadIdx.x == 0) cs = n > 0 ? __double2float_rn((double)a.alpha / (double)n) : 0.f;
     __syncthreads();
-    float r[8];
-    if (has_chunk) {
-      const float4 r0 = reinterpret_cast<const float4*>(Rs)[2 * sub];
-      const float4 r1 = reinterpret_cast<const float4*>(Rs)[2 * sub + 1];
-      r[0] = r0.x; r[1] = r0.y; r[2] = r0.z; r[3] = r0.w;
-      r[4] = r1.x; r[5] = r1.y; r[6] = r1.z; r[7] = r1.w;
-    } else {
+    // this lane's chunks: sub, sub + LPT, ... (CPL of them, past nch unused)
+    float r[CPL][8];
 #pragma unroll
-      for (int i = 0; i < 8; ++i) r[i] = 0.f;
+    for (int k = 0; k < CPL; ++k) {
+      const int c = sub + k * LPT;
+      if (c < nch) {
+        const float4 r0 = reinterpret_cast<const float4*>(Rs)[2 * c];
+        const float4 r1 = reinterpret_cast<const float4*>(Rs)[2 * c + 1];
+        r[k][0] = r0.x; r[k][1] = r0.y; r[k][2] = r0.z; r[k][3] = r0.w;
+        r[k][4] = r1.x; r[k][5] = r1.y; r[k][6] = r1.z; r[k][7] = r1.w;
+      } else {
+#pragma unroll
+        for (int i = 0; i < 8; ++i) r[k][i] = 0.f;
+      }
     }
     const float c0 = cs;
 
     for (int64_t base = t + (int64_t)wid * TPW; base < seg_end; base += (int64_t)nw * TPW) {
       const int64_t tok = base + slot;
-      const bool ok = has_chunk && tok < seg_end;
-      float s[8];
+      const bool tok_ok = tok < seg_end;
       float d = 0.f, num = 0.f;
-      if (ok) {
-        const uint4 w = __ldcs(reinterpret_cast<const uint4*>(a.z + tok * E) + sub);
-        const uint32_t zw[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-        for (int q = 0; q < 4; ++q) {
-          s[2 * q] = 1.0f / (1.0f + expf(-bf16_lo(zw[q])));
-          s[2 * q + 1] = 1.0f / (1.0f + expf(-bf16_hi(zw[q])));
-        }
+      for (int k = 0; k < CPL; ++k) {
+        const int c = sub + k * LPT;
+        if (tok_ok && c < nch) {
+          const uint4 w = __ldcs(reinterpret_cast<const uint4*>(a.z + tok * E) + c);
+          const uint32_t zw[4] = {w.x, w.y, w.z, w.w};
 #pragma unroll
-        for (int i = 0; i < 8; ++i) {
-          d = __fadd_rn(d, s[i]);
-          num = __fadd_rn(num, __fmul_rn(s[i], r[i]));
+          for (int q = 0; q < 4; ++q) {
+            const float s0 = 1.0f / (1.0f + expf(-bf16_lo(zw[q])));
+            const float s1 = 1.0f / (1.0f + expf(-bf16_hi(zw[q])));
+            d = __fadd_rn(d, s0);
+            num = __fadd_rn(num, __fmul_rn(s0, r[k][2 * q]));
+            d = __fadd_rn(d, s1);
+            num = __fadd_rn(num, __fmul_rn(s1, r[k][2 * q + 1]));
+          }
         }
       }
 #pragma unroll
@@ -81,19 +87,23 @@ __global__ void __launch_bounds__(kGsThreads) gshard_kernel(GshardArgs a, int64_
         d = __fadd_rn(d, __shfl_xor_sync(kFull, d, m));
         num = __fadd_rn(num, __shfl_xor_sync(kFull, num, m));
       }
-      if (ok) {
-        const float mean = __fdiv_rn(num, d);
-        const float coef = __fdiv_rn(c0, d);
-        float4* gp = reinterpret_cast<float4*>(a.g + tok * E) + 2 * sub;
+      if (!tok_ok) continue;
+      const float mean = __fdiv_rn(num, d);
+      const float coef = __fdiv_rn(c0, d);
+#pragma unroll
+      for (int k = 0; k < CPL; ++k) {
+        const int c = sub + k * LPT;
+        if (c >= nch) continue;
+        float4* gp = reinterpret_cast<float4*>(a.g + tok * E) + 2 * c;
         float4 g0 = __ldcs(gp), g1 = __ldcs(gp + 1);
-        g0.x = __fadd_rn(g0.x, __fmul_rn(coef, __fsub_rn(r[0], mean)));
-        g0.y = __fadd_rn(g0.y, __fmul_rn(coef, __fsub_rn(r[1], mean)));
-        g0.z = __fadd_rn(g0.z, __fmul_rn(coef, __fsub_rn(r[2], mean)));
-        g0.w = __fadd_rn(g0.w, __fmul_rn(coef, __fsub_rn(r[3], mean)));
-        g1.x = __fadd_rn(g1.x, __fmul_rn(coef, __fsub_rn(r[4], mean)));
-        g1.y = __fadd_rn(g1.y, __fmul_rn(coef, __fsub_rn(r[5], mean)));
-        g1.z = __fadd_rn(g1.z, __fmul_rn(coef, __fsub_rn(r[6], mean)));
-        g1.w = __fadd_rn(g1.w, __fmul_rn(coef, __fsub_rn(r[7], mean)));
+        g0.x = __fadd_rn(g0.x, __fmul_rn(coef, __fsub_rn(r[k][0], mean)));
+        g0.y = __fadd_rn(g0.y, __fmul_rn(coef, __fsub_rn(r[k][1], mean)));
+        g0.z = __fadd_rn(g0.z, __fmul_rn(coef, __fsub_rn(r[k][2], mean)));
+        g0.w = __fadd_rn(g0.w, __fmul_rn(coef, __fsub_rn(r[k][3], mean)));
+        g1.x = __fadd_rn(g1.x, __fmul_rn(coef, __fsub_rn(r[k][4], mean)));
+        g1.y = __fadd_rn(g1.y, __fmul_rn(coef, __fsub_rn(r[k][5], mean)));
+        g1.z = __fadd_rn(g1.z, __fmul_rn(coef, __fsub_rn(r[k][6], mean)));
+        g1.w = __fadd_rn(g1.w, __fmul_rn(coef, __fsub_rn(r[k][7], mean)));
         __stcs(gp, g0);
         __stcs(gp + 1, g1);
       }
@@ -102,7 +112,7 @@ __global__ void __launch_bounds__(kGsThreads) gshard_kernel(GshardArgs a, int64_
   }
 }
 
-template <int LPT>
+template <int LPT, int CPL>
 int launch_gs(const GshardArgs& a, cudaStream_t s) {
   DeviceInfo di;
   if (int rc = device_info(&di)) return rc;
@@ -111,7 +121,7 @@ int launch_gs(const GshardArgs& a, cudaStream_t s) {
   if (grid > max_grid) grid = max_grid;
   if (grid < 1) grid = 1;
   const int64_t tpc = (a.T + grid - 1) / grid;
-  gshard_kernel<LPT><<<(unsigned)grid, kGsThreads, 0, s>>>(a, tpc);
+  gshard_kernel<LPT, CPL><<<(unsigned)grid, kGsThreads, 0, s>>>(a, tpc);
   return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
 }
 
@@ -119,12 +129,15 @@ int launch_gs(const GshardArgs& a, cudaStream_t s) {
 
 int launch_gshard(const GshardArgs& a, cudaStream_t s) {
   const int nch = a.E >> 3;
-  if (nch <= 1) return launch_gs<1>(a, s);
-  if (nch <= 2) return launch_gs<2>(a, s);
-  if (nch <= 4) return launch_gs<4>(a, s);
-  if (nch <= 8) return launch_gs<8>(a, s);
-  if (nch <= 16) return launch_gs<16>(a, s);
-  if (nch <= 32) return launch_gs<32>(a, s);
+  if (nch <= 1) return launch_gs<1, 1>(a, s);
+  if (nch <= 2) return launch_gs<2, 1>(a, s);
+  if (nch <= 4) return launch_gs<4, 1>(a, s);
+  if (nch <= 8) return launch_gs<8, 1>(a, s);
+  if (nch <= 16) return launch_gs<16, 1>(a, s);
+  if (nch <= 32) return launch_gs<32, 1>(a, s);
+  if (nch <= 64) return launch_gs<32, 2>(a, s);
+  if (nch <= 96) return launch_gs<32, 3>(a, s);
+  if (nch <= 128) return launch_gs<32, 4>(a, s);
   return kErrUnsupported;
 }
 

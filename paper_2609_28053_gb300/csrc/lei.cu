@@ -9,9 +9,9 @@
 //
 // The path is a pure HBM stream (read and write grad_s once), so each CTA
 // takes a contiguous token range, computes the E coefficients of each
-// microbatch it meets (fp64, one thread per expert, a block max for xi) into
-// shared memory as fp32, and then streams its range with 16-byte loads and
-// stores using evict-first cache hints.
+// microbatch it meets (fp64, the threads striding over the experts, a block
+// max for xi) into shared memory as fp32, and then streams its range with
+// 16-byte loads and stores using evict-first cache hints.
 #include "eqb_device.cuh"
 
 namespace eqb {
@@ -22,7 +22,7 @@ constexpr int kLeiThreads = 256;
 constexpr int kLeiUnroll = 4;
 
 __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tokens_per_cta) {
-  __shared__ __align__(16) float coef[256];
+  __shared__ __align__(16) float coef[kMaxE];
   __shared__ double red[kLeiThreads / 32];
   __shared__ double scal[2];
   const int E = a.E, E4 = a.E >> 2;
@@ -51,10 +51,16 @@ __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tok
     }
     __syncthreads();
     const double inv_fbar = scal[0];
-    double rho = 0.0;
-    if (threadIdx.x < E && inv_fbar > 0.0)
-      rho = (double)__ldg(a.loads + (int64_t)l * E + threadIdx.x) * inv_fbar - 1.0;
-    double amax = fabs(rho);
+    // each thread holds the rho of experts threadIdx.x + k * blockDim.x
+    constexpr int kPer = kMaxE / kLeiThreads;
+    double rho[kPer];
+    double amax = 0.0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int e = threadIdx.x + k * kLeiThreads;
+      rho[k] = (e < E && inv_fbar > 0.0) ? (double)__ldg(a.loads + (int64_t)l * E + e) * inv_fbar - 1.0 : 0.0;
+      amax = fmax(amax, fabs(rho[k]));
+    }
 #pragma unroll
     for (int d = 16; d > 0; d >>= 1) amax = fmax(amax, __shfl_xor_sync(kFull, amax, d));
     if (lane == 0) red[wid] = amax;
@@ -70,7 +76,11 @@ __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tok
       scal[1] = (double)a.eta * sigma;
     }
     __syncthreads();
-    if (threadIdx.x < E) coef[threadIdx.x] = __double2float_rn(scal[1] * rho);
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+      const int e = threadIdx.x + k * kLeiThreads;
+      if (e < E) coef[e] = __double2float_rn(scal[1] * rho[k]);
+    }
     __syncthreads();
 
     // ---- stream grad_s[t .. seg_end) in float4 units

@@ -32,7 +32,6 @@ namespace eqb {
 
 namespace {
 
-constexpr int kEntries = 32;  // >= E/8 chunk entries per lane
 
 __host__ __device__ inline int row_stride_bytes(int E) {
   int w = E / 2;                     // 32-bit words per row
@@ -44,7 +43,7 @@ __host__ __device__ inline int align16(int x) { return (x + 15) & ~15; }
 __host__ __device__ inline int head_bytes(int E) { return align16(4 * E) + 2 * align16(2 * E); }
 
 __host__ __device__ inline int warp_region_bytes(int E, int nbuf) {
-  return align16(nbuf * 32 * row_stride_bytes(E) + kEntries * 32 * 2 + 4 * E);
+  return align16(nbuf * 32 * row_stride_bytes(E) + (E / 8) * 32 * 2 + 4 * E);  // tile, chunk lists, loads
 }
 
 template <int KP1, int G>
@@ -63,7 +62,7 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
   uint8_t* wreg = smem + head_bytes(E) + wid * warp_region_bytes(E, nbuf);
   uint8_t* tiles = wreg;
   uint16_t* ent = reinterpret_cast<uint16_t*>(wreg + nbuf * tile_bytes);
-  int* wl = reinterpret_cast<int*>(wreg + nbuf * tile_bytes + kEntries * 32 * 2);
+  int* wl = reinterpret_cast<int*>(wreg + nbuf * tile_bytes + nch * 32 * 2);
 
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
     const float v = a.b[e];
@@ -86,16 +85,16 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
   const uint4* bdn4 = reinterpret_cast<const uint4*>(bdn);
   const uint4* bup4 = reinterpret_cast<const uint4*>(bup);
 
-  // cp.async copies of one tile: row r, chunk `lane`.
+  // cp.async copies of one tile: row r, chunks lane, lane + 32, ...
   auto issue = [&](int64_t tile, int buf) {
     uint8_t* dst = tiles + buf * tile_bytes;
     const int64_t t0 = tile << 5;
-    if (lane < nch) {
+    for (int c = lane; c < nch; c += 32) {
 #pragma unroll 4
       for (int r = 0; r < 32; ++r) {
         const bool ok = t0 + r < a.T;
-        const uint16_t* src = ok ? a.z + (t0 + r) * E + lane * 8 : a.z;
-        cp_async16(dst + r * rs + lane * 16, src, ok ? 16 : 0);
+        const uint16_t* src = ok ? a.z + (t0 + r) * E + c * 8 : a.z;
+        cp_async16(dst + r * rs + c * 16, src, ok ? 16 : 0);
       }
     }
   };

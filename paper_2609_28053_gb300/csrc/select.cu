@@ -85,10 +85,10 @@ __device__ __forceinline__ void bf16_exp_range(uint32_t x, int& lo, int& hi) {
 
 // b_next = q_hat - mean(q_hat), mean = (sum in ascending e, fp64) / E.
 // If every non-zero q_hat lies within a window where all partial sums of up
-// to 256 terms are exact in fp64 (leading-bit exponent - ulp exponent + 9 <=
-// 52), any summation order gives the exact sum, so a warp tree reduction
-// reproduces the sequential sum bit for bit.  Otherwise one thread sums in
-// ascending order.
+// to E terms are exact in fp64 (leading-bit exponent - ulp exponent + 1 +
+// ceil(log2 E) <= 52), any summation order gives the exact sum, so a warp
+// tree reduction reproduces the sequential sum bit for bit.  Otherwise one
+// thread sums in ascending order.
 __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, float* __restrict__ b_next) {
   __shared__ double mean;
   if (threadIdx.x < 32) {
@@ -111,7 +111,8 @@ __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, fl
       hi = max(hi, __shfl_xor_sync(kFull, hi, d));
     }
     double sum;
-    if (hi - lo + 9 <= 52 || hi < lo) {
+    const int lg = 32 - __clz(E - 1);  // ceil(log2 E)
+    if (hi - lo + 1 + lg <= 52 || hi < lo) {
 #pragma unroll
       for (int d = 16; d > 0; d >>= 1) part = __dadd_rn(part, __shfl_xor_sync(kFull, part, d));
       sum = part;

@@ -60,7 +60,7 @@ eqb_status check_step(const eqb_bf16* z, const float* b, int64_t T, int32_t E, i
                       float eta, float c, void* workspace, size_t workspace_bytes, int32_t* err_flag,
                       Workspace* w) {
   if (T < 1 || E < 2 || K < 1 || K >= E || M < 1) return EQB_ERR_INVALID_ARG;
-  if (E > 256 || (E % 8) != 0 || K + 1 > 32) return EQB_ERR_UNSUPPORTED;
+  if (E > eqb::kMaxE || (E % 8) != 0 || K + 1 > 32) return EQB_ERR_UNSUPPORTED;
   if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
   if (!z || !b || !mb_offsets || !tau || !loads || !b_next || !workspace) return EQB_ERR_INVALID_ARG;
   if (grad_s && (!(eta == eta) || !(c == c))) return EQB_ERR_INVALID_ARG;

@@ -69,7 +69,7 @@ def route(lib, z=FAKE, b=FAKE, T=64, E=64, K=8, off=FAKE, M=1, idx=FAKE, tau=FAK
 
 @pytest.mark.parametrize("kw,code", [
     (dict(K=0), INVALID), (dict(K=64), INVALID), (dict(T=-1), INVALID), (dict(E=1), INVALID),
-    (dict(E=12), UNSUPPORTED), (dict(E=264), UNSUPPORTED), (dict(E=64, K=32), UNSUPPORTED),
+    (dict(E=12), UNSUPPORTED), (dict(E=1032), UNSUPPORTED), (dict(E=64, K=32), UNSUPPORTED),
     (dict(T=1 << 31), UNSUPPORTED), (dict(z=NULL), INVALID), (dict(b=NULL), INVALID),
     (dict(tau=NULL), INVALID), (dict(off=NULL), INVALID), (dict(M=0), INVALID),
     (dict(z=MISALIGNED), INVALID), (dict(tau=MISALIGNED), INVALID),
@@ -93,7 +93,7 @@ def test_hist_and_select_reject(lib):
     assert lib.eqb_select_quantile(FAKE, 64, 2, 5, FAKE, FAKE, NULL, NULL, NULL) == INVALID
     assert lib.eqb_select_quantile(FAKE, 300, 1, 5, FAKE, FAKE, NULL, NULL, NULL) == UNSUPPORTED
     assert lib.eqb_bias_update(FAKE, 0, FAKE, NULL) == INVALID
-    assert lib.eqb_bias_update(FAKE, 257, FAKE, NULL) == UNSUPPORTED
+    assert lib.eqb_bias_update(FAKE, 1025, FAKE, NULL) == UNSUPPORTED
 
 
 def test_lei_rejects(lib):
@@ -211,7 +211,7 @@ def test_gshard_rejects(lib):
     f = lib.gshard_inject_grad
     a = ctypes.c_float(0.01)
     assert f(FAKE, FAKE, FAKE, FAKE, 2, 10, 12, 2, a, NULL) == UNSUPPORTED     # E % 8
-    assert f(FAKE, FAKE, FAKE, FAKE, 2, 10, 264, 2, a, NULL) == UNSUPPORTED    # E > 256
+    assert f(FAKE, FAKE, FAKE, FAKE, 2, 10, 1032, 2, a, NULL) == UNSUPPORTED   # E > 1024
     assert f(NULL, FAKE, FAKE, FAKE, 2, 10, 64, 2, a, NULL) == INVALID
     assert f(MISALIGNED, FAKE, FAKE, FAKE, 2, 10, 64, 2, a, NULL) == INVALID
     assert f(FAKE, FAKE, FAKE, FAKE, 2, 10, 64, 2, ctypes.c_float(float("nan")), NULL) == INVALID
@@ -233,7 +233,7 @@ def test_comparison_statistics_reject(lib):
     assert ra(off=None) == INVALID
     assert ra(q=NULL) == INVALID
     assert ra(wsb=ws - 1) == INVALID
-    assert ra(E=72 + 200) == UNSUPPORTED
+    assert ra(E=1032) == UNSUPPORTED
     g = lib.eqb_fixed_hist_bias
     fl = ctypes.c_float
     assert g(FAKE, FAKE, 100, 64, 8, fl(-1.0), fl(0.0), FAKE, NULL, FAKE, ws, NULL, NULL) == INVALID

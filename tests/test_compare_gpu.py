@@ -32,7 +32,8 @@ def workspace(E):
 
 
 @pytest.mark.parametrize("T,E,K,shards", [(4000, 64, 8, [0, 1000, 1000, 2500, 4000]), (3001, 16, 2, [0, 3001]),
-                                          (20000, 256, 8, list(range(0, 20001, 2500))), (5000, 128, 6, [0, 7, 5000])])
+                                          (20000, 256, 8, list(range(0, 20001, 2500))), (5000, 128, 6, [0, 7, 5000]),
+                                          (3000, 384, 8, [0, 1500, 3000])])
 def test_rank_averaged_bias_matches_oracle(T, E, K, shards):
     z, tau = case(T, E, K, seed=T + E)
     want_b, want_q = oracle.rank_averaged_bias(z, tau, K, shards)
@@ -50,7 +51,8 @@ def test_rank_averaged_bias_matches_oracle(T, E, K, shards):
 
 
 @pytest.mark.parametrize("T,E,K,lo,width", [(4000, 64, 8, -4.0, 1.0 / 32), (3001, 16, 2, -1.0, 0.01),
-                                            (20000, 256, 8, -8.0, 0.0625), (5000, 128, 6, 0.5, 0.1)])
+                                            (20000, 256, 8, -8.0, 0.0625), (5000, 128, 6, 0.5, 0.1),
+                                            (3000, 1024, 8, -6.0, 0.05)])
 def test_fixed_hist_bias_matches_oracle(T, E, K, lo, width):
     """Includes ranges that clamp many margins into the edge bins."""
     z, tau = case(T, E, K, seed=T * 3 + E)

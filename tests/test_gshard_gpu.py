@@ -41,7 +41,8 @@ def bound(z_bits, loads, off, K, alpha, g_ref):
 
 
 @pytest.mark.parametrize("T,E,K,M", [(1, 8, 2, 1), (1000, 64, 8, 5), (777, 24, 3, 3), (4099, 256, 8, 7),
-                                     (3000, 128, 6, 4), (500, 40, 4, 2)])
+                                     (3000, 128, 6, 4), (500, 40, 4, 2), (777, 512, 8, 3), (300, 1024, 6, 2),
+                                     (400, 264, 4, 2)])
 @pytest.mark.parametrize("alpha", [1e-2, 3.0])
 def test_gshard_matches_oracle(T, E, K, M, alpha):
     rng = np.random.default_rng(T + E + K)
