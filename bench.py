@@ -344,8 +344,9 @@ def extras(step, stream, peak):
     mv = torch.empty(2, dtype=torch.float64, device=dev)
     out["maxvio"] = {"ms": round(time_call(lambda: eqb.eqb_maxvio(step.loads, off, K, out=mv, stream=stream),
                                            stream), 5)}
+    ws_ra = torch.zeros(eqb.eqb_rank_averaged_workspace_bytes(E, M), dtype=torch.uint8, device=dev)
     row("rank_averaged_bias", time_call(lambda: eqb.eqb_rank_averaged_bias(
-        z, step.tau, K, shards, step.workspace, stream=stream), stream, reps=3), 2 * (2 * T * E + 4 * T))
+        z, step.tau, K, shards, ws_ra, stream=stream), stream, reps=3), 2 * (2 * T * E + 4 * T))
     row("fixed_hist_bias", time_call(lambda: eqb.eqb_fixed_hist_bias(
         z, step.tau, K, lo, width, step.workspace, stream=stream), stream), 2 * T * E + 4 * T)
 
@@ -356,7 +357,7 @@ def extras(step, stream, peak):
     eqb.eqb_layer_step(z, b0, K, off, loads, step.b_next, step.workspace, tau=tau, mb_offsets_host=step.off_h,
                        stream=stream)
     biases = {"before": b0, "eqb": step.b_next.clone(),
-              "rank_averaged": eqb.eqb_rank_averaged_bias(z, tau, K, shards, step.workspace, stream=stream)[0].clone(),
+              "rank_averaged": eqb.eqb_rank_averaged_bias(z, tau, K, shards, ws_ra, stream=stream)[0].clone(),
               "fixed_hist": eqb.eqb_fixed_hist_bias(z, tau, K, lo, width, step.workspace, stream=stream)[0].clone()}
     fresh = make_logits(step.workload, T=T, seed=SHAPES[step.workload].seed + 977, device=str(dev))
     bal = {}
@@ -366,6 +367,30 @@ def extras(step, stream, peak):
         eqb.eqb_maxvio(loads, off, K, out=mv, stream=stream)
         g_, l_ = mv.tolist()
         bal[name] = {"maxvio_global": round(g_, 4), "maxvio_local": round(l_, 4)}
+    # The oracle on a bounded sample of the same workload, one host core.
+    import oracle
+    from eqb_workloads import bits
+    n = min(16384, T)
+    per = max(1, T // M)
+    zb = bits(z[:n])
+    b_h = step.b.cpu().numpy()
+    off_n = even_offsets(n, max(1, n // per)) if n >= per else np.array([0, n], np.int64)
+    _, tau_n, loads_n = oracle.route(zb, b_h, K, off_n)
+    g_n = step.g[:n].cpu().numpy()
+    shards_n = even_offsets(n, 4)
+
+    def ocpu(name, fn):
+        t0 = time.perf_counter()
+        fn()
+        secs = time.perf_counter() - t0
+        out[name]["cpu_oracle"] = {"tokens_per_s": round(n / secs, 1), "sample_tokens": n, "cores": 1,
+                                   "seconds": round(secs, 3)}
+
+    ocpu("gshard_inject_grad", lambda: oracle.gshard(g_n, zb, loads_n, off_n, K, 1e-2))
+    ocpu("maxvio", lambda: oracle.maxvio(loads_n, off_n, K))
+    ocpu("rank_averaged_bias", lambda: oracle.rank_averaged_bias(zb, tau_n, K, shards_n))
+    ocpu("fixed_hist_bias", lambda: oracle.fixed_hist_bias(zb, tau_n, K, lo, width))
+
     out["maxvio_after_one_update"] = {
         "batch": f"fresh {step.workload} batch, seed +977; biases from the timed batch",
         "rank_averaged_shards": M, "fixed_hist_bins": f"256 x {width} from {lo}", **bal}

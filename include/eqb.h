@@ -242,19 +242,22 @@ eqb_status gshard_inject_grad(float *grad_s, const eqb_bf16 *z, const int32_t *l
  * Both take the margins m = bf16_rne(tau_t - fp32(z_{t,e})) of
  * eqb_margin_hist_pass1 (so tau comes from eqb_route_topk), end with the
  * Eq. (2) centering b_e = fp32(x_e - mean(x)) (fp64, mean summed in ascending
- * expert order), and use a workspace of eqb_layer_workspace_bytes(E) bytes
- * (256-byte aligned).  Supported: E a multiple of 8, E <= 1024, T >= 1.
+ * expert order), and use a caller-provided workspace (256-byte aligned).
+ * Supported: E a multiple of 8, E <= 1024, T >= 1.
  *
  * Rank-averaged QB: every shard p (token range [offsets[p], offsets[p+1]))
  * selects its own K/E quantile exactly (the r_p-th smallest margin,
  * r_p = ceil(n_p K / E), by the same two radix passes as EQB); x_e is the
  * mean over the non-empty shards of those quantiles (fp64, summed in
- * ascending shard order).
- *   shard_offsets_host  host int64 [P+1], 0 = first <= ... <= last = T
- *   q_shards            device bf16 [P,E] (out): the non-empty shards'
- *                       quantiles in rows 0.. in shard order
+ * ascending shard order).  Its workspace is
+ * eqb_rank_averaged_workspace_bytes(E, P) bytes (per-shard histograms).
+ *   shard_offsets_host  host int64 [P+1], 0 = first <= ... <= last = T,
+ *                       1 <= P <= 65535
+ *   q_shards            device bf16 [P,E] (out): row p holds shard p's
+ *                       quantiles (+0 for an empty shard)
  *   err_flag            as in eqb_select_quantile
  * The result depends on how the tokens are sharded; EQB's does not. */
+size_t eqb_rank_averaged_workspace_bytes(int32_t E, int32_t P);
 eqb_status eqb_rank_averaged_bias(const eqb_bf16 *z, const float *tau, int64_t T, int32_t E,
                                   int32_t K, const int64_t *shard_offsets_host, int32_t P,
                                   eqb_bf16 *q_shards, float *b_out, void *workspace,
@@ -264,7 +267,8 @@ eqb_status eqb_rank_averaged_bias(const eqb_bf16 *z, const float *tau, int64_t T
  * in bin j = floor(fp32(fp32(m - lo) * fp32(1 / width))) clamped to
  * [0, 255]; x_e = lo + (j_e + 1) * width (fp64), the upper edge of the first
  * bin whose cumulative count reaches r = ceil(T K / E).  Its resolution is
- * the bin width, the limitation EQB removes.
+ * the bin width, the limitation EQB removes.  Its workspace is
+ * eqb_layer_workspace_bytes(E) bytes.
  *   lo, width   finite, width > 0
  *   estimate    device double [E] (out, nullable): x before centering */
 eqb_status eqb_fixed_hist_bias(const eqb_bf16 *z, const float *tau, int64_t T, int32_t E,

@@ -33,6 +33,7 @@ __all__ = [
     "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route", "eqb_router_layer_step",
     "eqb_maxvio", "gshard_inject_grad", "eqb_rank_averaged_bias", "eqb_fixed_hist_bias",
+    "eqb_rank_averaged_workspace_bytes",
 ]
 
 
@@ -202,11 +203,17 @@ def gshard_inject_grad(grad_s, z, loads, mb_offsets, K, alpha, stream=None):
     return grad_s
 
 
+def eqb_rank_averaged_workspace_bytes(E: int, P: int) -> int:
+    return int(load().eqb_rank_averaged_workspace_bytes(E, P))
+
+
 def eqb_rank_averaged_bias(z, tau, K, shard_offsets_host, workspace, b_out=None, q_shards=None,
                            err_flag=None, stream=None):
     """Rank-averaged QB (Sec. 2): each shard's own K/E margin quantile,
     averaged over the non-empty shards and centered.  shard_offsets_host: int64
-    host array [P+1].  Returns (b fp32 [E], q_shards bf16 [P,E])."""
+    host array [P+1]; workspace: uint8 CUDA tensor of
+    eqb_rank_averaged_workspace_bytes(E, P) bytes.  Returns (b fp32 [E],
+    q_shards bf16 [P,E], row p = shard p)."""
     import numpy as np
     T, E = z.shape
     _need(z, torch.bfloat16, "z")

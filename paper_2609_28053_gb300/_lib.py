@@ -18,7 +18,7 @@ EXPORTS = (
     "eqb_bias_update", "lei_inject_grad", "eqb_router_logits", "eqb_layer_workspace_bytes",
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route",
     "eqb_router_layer_step", "eqb_maxvio", "gshard_inject_grad",
-    "eqb_rank_averaged_bias", "eqb_fixed_hist_bias",
+    "eqb_rank_averaged_bias", "eqb_fixed_hist_bias", "eqb_rank_averaged_workspace_bytes",
 )
 
 STATUS = {0: "EQB_OK", 1: "EQB_ERR_INVALID_ARG", 2: "EQB_ERR_UNSUPPORTED", 3: "EQB_ERR_CUDA",
@@ -76,6 +76,8 @@ def load(path: str | None = None) -> ctypes.CDLL:
         lib.eqb_version.restype = ctypes.c_int
         lib.eqb_layer_workspace_bytes.argtypes = [i32]
         lib.eqb_layer_workspace_bytes.restype = ctypes.c_size_t
+        lib.eqb_rank_averaged_workspace_bytes.argtypes = [i32, i32]
+        lib.eqb_rank_averaged_workspace_bytes.restype = ctypes.c_size_t
         lib.eqb_target_rank.argtypes = [i64, i32, i32]
         lib.eqb_target_rank.restype = i64
         if path is None:

@@ -52,6 +52,10 @@ struct HistArgs {
   int32_t* hist;
   int32_t* err;
   float lo = 0.f, inv_w = 0.f;  // pass 3 (equal-width bins) only
+  // Optional token shards (device int64 [P+1]): shard p's counts go to
+  // hist + p*E*256, and pass 2 takes shard p's selected bins from u + p*E.
+  const int64_t* shard_off = nullptr;
+  int P = 0;
 };
 
 struct LeiArgs {
@@ -94,6 +98,11 @@ int launch_route_wide(const RouteArgs& a, cudaStream_t s);
 int launch_hist(const HistArgs& a, int pass, cudaStream_t s);
 int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, int32_t* rho,
                   uint16_t* q_hat, int32_t* err, cudaStream_t s);
+// One selection per token shard (device int64 [P+1]): shard p reads
+// hist + p*E*256 and writes u, rho, q_hat + p*E at its own rank
+// ceil(n_p K / E); an empty shard gets u = rho = 0 and q_hat = +0.
+int launch_select_sharded(const int32_t* hist, int E, int pass, const int64_t* shard_off, int P, int K,
+                          uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err, cudaStream_t s);
 int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t s);
 int launch_lei(const LeiArgs& a, cudaStream_t s);
 int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, uint16_t* z,

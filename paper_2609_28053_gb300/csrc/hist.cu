@@ -58,16 +58,17 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
   const uint32_t base = static_cast<uint32_t>(__cvta_generic_to_shared(bins)) +
                         4u * static_cast<uint32_t>(Lay::row_word(4 * c));
   uint32_t sel[4] = {0, 0, 0, 0};
-  if (PASS == 2) {
-    // internal high bytes (u ^ 0x80) of the selected bins, placed where the
-    // internal keys carry them: bits 8-15 (even expert) and 24-31 (odd).
+  // internal high bytes (u ^ 0x80) of the selected bins, placed where the
+  // internal keys carry them: bits 8-15 (even expert) and 24-31 (odd).
+  auto load_sel = [&](const uint8_t* ub) {
 #pragma unroll
     for (int p = 0; p < 4; ++p) {
-      const uint32_t ue = a.u[e0 + c * 8 + 2 * p] ^ 0x80u;
-      const uint32_t uo = a.u[e0 + c * 8 + 2 * p + 1] ^ 0x80u;
+      const uint32_t ue = ub[e0 + c * 8 + 2 * p] ^ 0x80u;
+      const uint32_t uo = ub[e0 + c * 8 + 2 * p + 1] ^ 0x80u;
       sel[p] = (ue << 8) | (uo << 24);
     }
-  }
+  };
+  if (PASS == 2 && !a.shard_off) load_sel(a.u);
   __syncthreads();
 
   // Token indices fit in 32 bits (T < 2^31 is checked on the host).
@@ -105,8 +106,16 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
     }
   };
 
-  for (int cb = tb; cb < te; cb += static_cast<int>(kFlushTokens)) {
-    const int ce = static_cast<int>(min((int64_t)cb + kFlushTokens, (int64_t)te));
+  for (int cb = tb; cb < te;) {
+    int ce = static_cast<int>(min((int64_t)cb + kFlushTokens, (int64_t)te));
+    int64_t hbase = 0;  // this chunk's histogram (shards: one per shard)
+    if (a.shard_off) {
+      const int sp = microbatch_of(a.shard_off, a.P, cb);
+      const int64_t send = __ldg(a.shard_off + sp + 1);
+      if (send > cb && send < ce) ce = static_cast<int>(send);  // chunks end at shard boundaries
+      hbase = (int64_t)sp * E * 256;
+      if (PASS == 2) load_sel(a.u + (int64_t)sp * E);
+    }
     int t = cb + wid * Lay::TPS + tok;
     const uint16_t* zp = zlane + static_cast<size_t>(t) * E;
     // full rounds of kUnroll tokens per lane, no guards
@@ -136,12 +145,13 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
         bins[wi] = 0u;
         const int bin = (PASS == 1) ? (slot ^ 0x80) : slot;  // pass 1 stores internal keys
         const int ee = e0 + 2 * row;
-        if (v & 0xffffu) atomicAdd(a.hist + (int64_t)ee * 256 + bin, static_cast<int>(v & 0xffffu));
-        if (v >> 16) atomicAdd(a.hist + (int64_t)(ee + 1) * 256 + bin, static_cast<int>(v >> 16));
+        if (v & 0xffffu) atomicAdd(a.hist + hbase + (int64_t)ee * 256 + bin, static_cast<int>(v & 0xffffu));
+        if (v >> 16) atomicAdd(a.hist + hbase + (int64_t)(ee + 1) * 256 + bin, static_cast<int>(v >> 16));
         if (PASS == 1 && (bin == 0 || bin == 255)) raise_flag(a.err, kErrNonfinite);
       }
     }
     __syncthreads();
+    cb = ce;
   }
 }
 

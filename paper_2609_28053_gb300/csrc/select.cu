@@ -22,10 +22,28 @@ namespace {
 __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__ hist, int E, int pass,
                                                      int64_t r, uint8_t* __restrict__ u,
                                                      int32_t* __restrict__ rho,
-                                                     uint16_t* __restrict__ q_hat, int32_t* err) {
+                                                     uint16_t* __restrict__ q_hat, int32_t* err,
+                                                     const int64_t* __restrict__ shard_off, int K) {
   const int lane = threadIdx.x & 31;
   const int e = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (e >= E) return;
+  if (shard_off) {
+    // shard blockIdx.y: its own histogram, outputs and rank ceil(n_p K / E)
+    const int p = blockIdx.y;
+    const int64_t n = shard_off[p + 1] - shard_off[p];
+    hist += (int64_t)p * E * 256;
+    u += (int64_t)p * E;
+    rho += (int64_t)p * E;
+    if (q_hat) q_hat += (int64_t)p * E;
+    if (n <= 0) {
+      if (lane == 0) {
+        if (pass != 2) { u[e] = 0; rho[e] = 0; }
+        else q_hat[e] = 0;
+      }
+      return;
+    }
+    r = (n * K + E - 1) / E;
+  }
   const int32_t* h = hist + (int64_t)e * 256 + lane * 8;
   int64_t cnt[8];
   int64_t local = 0;
@@ -133,7 +151,15 @@ __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, fl
 int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, int32_t* rho,
                   uint16_t* q_hat, int32_t* err, cudaStream_t s) {
   const int wpb = 8;
-  select_kernel<<<(E + wpb - 1) / wpb, wpb * 32, 0, s>>>(hist, E, pass, r, u, rho, q_hat, err);
+  select_kernel<<<(E + wpb - 1) / wpb, wpb * 32, 0, s>>>(hist, E, pass, r, u, rho, q_hat, err, nullptr, 0);
+  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+}
+
+int launch_select_sharded(const int32_t* hist, int E, int pass, const int64_t* shard_off, int P, int K,
+                          uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err, cudaStream_t s) {
+  const int wpb = 8;
+  dim3 grid((E + wpb - 1) / wpb, P);
+  select_kernel<<<grid, wpb * 32, 0, s>>>(hist, E, pass, 0, u, rho, q_hat, err, shard_off, K);
   return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
 }
 

@@ -221,7 +221,8 @@ def test_gshard_rejects(lib):
 
 def test_comparison_statistics_reject(lib):
     import numpy as np
-    ws = lib.eqb_layer_workspace_bytes(64)
+    ws = lib.eqb_rank_averaged_workspace_bytes(64, 2)
+    assert ws >= 2 * 2 * 64 * 256 * 4
     good = np.array([0, 40, 100], np.int64)
     bad = np.array([0, 60, 50], np.int64)
     f = lib.eqb_rank_averaged_bias
@@ -234,6 +235,7 @@ def test_comparison_statistics_reject(lib):
     assert ra(q=NULL) == INVALID
     assert ra(wsb=ws - 1) == INVALID
     assert ra(E=1032) == UNSUPPORTED
+    ws = lib.eqb_layer_workspace_bytes(64)
     g = lib.eqb_fixed_hist_bias
     fl = ctypes.c_float
     assert g(FAKE, FAKE, 100, 64, 8, fl(-1.0), fl(0.0), FAKE, NULL, FAKE, ws, NULL, NULL) == INVALID

@@ -33,7 +33,8 @@ def workspace(E):
 
 @pytest.mark.parametrize("T,E,K,shards", [(4000, 64, 8, [0, 1000, 1000, 2500, 4000]), (3001, 16, 2, [0, 3001]),
                                           (20000, 256, 8, list(range(0, 20001, 2500))), (5000, 128, 6, [0, 7, 5000]),
-                                          (3000, 384, 8, [0, 1500, 3000])])
+                                          (3000, 384, 8, [0, 1500, 3000]),
+                                          (70000, 256, 8, [0] + sorted(np.random.default_rng(9).integers(0, 70000, 39).tolist()) + [70000])])
 def test_rank_averaged_bias_matches_oracle(T, E, K, shards):
     z, tau = case(T, E, K, seed=T + E)
     want_b, want_q = oracle.rank_averaged_bias(z, tau, K, shards)
@@ -41,12 +42,15 @@ def test_rank_averaged_bias_matches_oracle(T, E, K, shards):
     B = Guarded((E,), torch.float32)
     Q = Guarded((P, E), torch.bfloat16, canary=-5.0)
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
-    eqb.eqb_rank_averaged_bias(to_dev_bf16(z), torch.from_numpy(tau).cuda(), K, np.array(shards), workspace(E),
+    ws = torch.zeros(eqb.eqb_rank_averaged_workspace_bytes(E, P), dtype=torch.uint8, device="cuda")
+    eqb.eqb_rank_averaged_bias(to_dev_bf16(z), torch.from_numpy(tau).cuda(), K, np.array(shards), ws,
                                b_out=B.view, q_shards=Q.view, err_flag=err)
     torch.cuda.synchronize()
     assert B.intact() and Q.intact() and err.item() == 0
     q = Q.view.view(torch.int16).cpu().numpy().view(np.uint16)
-    assert np.array_equal(q[:len(want_q)], want_q)
+    nonempty = [p for p in range(P) if shards[p + 1] > shards[p]]
+    assert np.array_equal(q[nonempty], want_q)
+    assert np.all(q[[p for p in range(P) if p not in nonempty]] == 0)
     assert np.array_equal(B.view.cpu().numpy().view(np.uint32), want_b.view(np.uint32))
 
 
@@ -78,7 +82,9 @@ def test_partition_invariance_eqb_vs_rank_average():
     zd, td = to_dev_bf16(z), torch.from_numpy(tau).cuda()
     outs = []
     for shards in ([0, T], list(range(0, T + 1, 8192)), [0, 5000, 30000, 30000, T]):
-        bq, _ = eqb.eqb_rank_averaged_bias(zd, td, K, np.array(shards), workspace(E))
+        ws = torch.zeros(eqb.eqb_rank_averaged_workspace_bytes(E, len(shards) - 1), dtype=torch.uint8,
+                         device="cuda")
+        bq, _ = eqb.eqb_rank_averaged_bias(zd, td, K, np.array(shards), ws)
         outs.append(bq.cpu().numpy())
     torch.cuda.synchronize()
     # one shard is EQB itself
