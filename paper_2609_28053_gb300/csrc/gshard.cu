@@ -61,51 +61,73 @@ __global__ void __launch_bounds__(kGsThreads) gshard_kernel(GshardArgs a, int64_
     }
     const float c0 = cs;
 
-    for (int64_t base = t + (int64_t)wid * TPW; base < seg_end; base += (int64_t)nw * TPW) {
-      const int64_t tok = base + slot;
-      const bool tok_ok = tok < seg_end;
-      float d = 0.f, num = 0.f;
+    // Two tokens per lane per round, every load issued before any use, so
+    // the z and grad loads of both overlap.
+    const int64_t stride = (int64_t)nw * TPW;
+    for (int64_t base = t + (int64_t)wid * TPW; base < seg_end; base += 2 * stride) {
+      int64_t tok[2];
+      bool ok[2];
+      uint4 w[2][CPL];
+      float4 g0[2][CPL], g1[2][CPL];
 #pragma unroll
-      for (int k = 0; k < CPL; ++k) {
-        const int c = sub + k * LPT;
-        if (tok_ok && c < nch) {
-          const uint4 w = __ldcs(reinterpret_cast<const uint4*>(a.z + tok * E) + c);
-          const uint32_t zw[4] = {w.x, w.y, w.z, w.w};
+      for (int u = 0; u < 2; ++u) {
+        tok[u] = base + u * stride + slot;
+        ok[u] = tok[u] < seg_end;
 #pragma unroll
-          for (int q = 0; q < 4; ++q) {
-            const float s0 = 1.0f / (1.0f + expf(-bf16_lo(zw[q])));
-            const float s1 = 1.0f / (1.0f + expf(-bf16_hi(zw[q])));
-            d = __fadd_rn(d, s0);
-            num = __fadd_rn(num, __fmul_rn(s0, r[k][2 * q]));
-            d = __fadd_rn(d, s1);
-            num = __fadd_rn(num, __fmul_rn(s1, r[k][2 * q + 1]));
+        for (int k = 0; k < CPL; ++k) {
+          const int c = sub + k * LPT;
+          if (ok[u] && c < nch) {
+            w[u][k] = __ldcs(reinterpret_cast<const uint4*>(a.z + tok[u] * E) + c);
+            const float4* gp = reinterpret_cast<const float4*>(a.g + tok[u] * E) + 2 * c;
+            g0[u][k] = __ldcs(gp);
+            g1[u][k] = __ldcs(gp + 1);
           }
         }
       }
 #pragma unroll
-      for (int m = 1; m < LPT; m <<= 1) {
-        d = __fadd_rn(d, __shfl_xor_sync(kFull, d, m));
-        num = __fadd_rn(num, __shfl_xor_sync(kFull, num, m));
-      }
-      if (!tok_ok) continue;
-      const float mean = __fdiv_rn(num, d);
-      const float coef = __fdiv_rn(c0, d);
+      for (int u = 0; u < 2; ++u) {
+        float d = 0.f, num = 0.f;
 #pragma unroll
-      for (int k = 0; k < CPL; ++k) {
-        const int c = sub + k * LPT;
-        if (c >= nch) continue;
-        float4* gp = reinterpret_cast<float4*>(a.g + tok * E) + 2 * c;
-        float4 g0 = __ldcs(gp), g1 = __ldcs(gp + 1);
-        g0.x = __fadd_rn(g0.x, __fmul_rn(coef, __fsub_rn(r[k][0], mean)));
-        g0.y = __fadd_rn(g0.y, __fmul_rn(coef, __fsub_rn(r[k][1], mean)));
-        g0.z = __fadd_rn(g0.z, __fmul_rn(coef, __fsub_rn(r[k][2], mean)));
-        g0.w = __fadd_rn(g0.w, __fmul_rn(coef, __fsub_rn(r[k][3], mean)));
-        g1.x = __fadd_rn(g1.x, __fmul_rn(coef, __fsub_rn(r[k][4], mean)));
-        g1.y = __fadd_rn(g1.y, __fmul_rn(coef, __fsub_rn(r[k][5], mean)));
-        g1.z = __fadd_rn(g1.z, __fmul_rn(coef, __fsub_rn(r[k][6], mean)));
-        g1.w = __fadd_rn(g1.w, __fmul_rn(coef, __fsub_rn(r[k][7], mean)));
-        __stcs(gp, g0);
-        __stcs(gp + 1, g1);
+        for (int k = 0; k < CPL; ++k) {
+          const int c = sub + k * LPT;
+          if (ok[u] && c < nch) {
+            const uint32_t zw[4] = {w[u][k].x, w[u][k].y, w[u][k].z, w[u][k].w};
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const float s0 = 1.0f / (1.0f + expf(-bf16_lo(zw[q])));
+              const float s1 = 1.0f / (1.0f + expf(-bf16_hi(zw[q])));
+              d = __fadd_rn(d, s0);
+              num = __fadd_rn(num, __fmul_rn(s0, r[k][2 * q]));
+              d = __fadd_rn(d, s1);
+              num = __fadd_rn(num, __fmul_rn(s1, r[k][2 * q + 1]));
+            }
+          }
+        }
+#pragma unroll
+        for (int m = 1; m < LPT; m <<= 1) {
+          d = __fadd_rn(d, __shfl_xor_sync(kFull, d, m));
+          num = __fadd_rn(num, __shfl_xor_sync(kFull, num, m));
+        }
+        if (!ok[u]) continue;
+        const float mean = __fdiv_rn(num, d);
+        const float coef = __fdiv_rn(c0, d);
+#pragma unroll
+        for (int k = 0; k < CPL; ++k) {
+          const int c = sub + k * LPT;
+          if (c >= nch) continue;
+          float4 x0 = g0[u][k], x1 = g1[u][k];
+          x0.x = __fadd_rn(x0.x, __fmul_rn(coef, __fsub_rn(r[k][0], mean)));
+          x0.y = __fadd_rn(x0.y, __fmul_rn(coef, __fsub_rn(r[k][1], mean)));
+          x0.z = __fadd_rn(x0.z, __fmul_rn(coef, __fsub_rn(r[k][2], mean)));
+          x0.w = __fadd_rn(x0.w, __fmul_rn(coef, __fsub_rn(r[k][3], mean)));
+          x1.x = __fadd_rn(x1.x, __fmul_rn(coef, __fsub_rn(r[k][4], mean)));
+          x1.y = __fadd_rn(x1.y, __fmul_rn(coef, __fsub_rn(r[k][5], mean)));
+          x1.z = __fadd_rn(x1.z, __fmul_rn(coef, __fsub_rn(r[k][6], mean)));
+          x1.w = __fadd_rn(x1.w, __fmul_rn(coef, __fsub_rn(r[k][7], mean)));
+          float4* gp = reinterpret_cast<float4*>(a.g + tok[u] * E) + 2 * c;
+          __stcs(gp, x0);
+          __stcs(gp + 1, x1);
+        }
       }
     }
     t = seg_end;
