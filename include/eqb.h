@@ -335,6 +335,16 @@ eqb_status eqb_router_layer_step(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t
                                  float eta, float c, void *workspace, size_t workspace_bytes,
                                  int32_t *err_flag, void *stream);
 
+/* Self-test of failure detection (no GPU fault involved): every wait in the
+ * library's kernels is a bounded poll of a shared-memory mbarrier, and a
+ * kernel whose pipeline stalls gives up, writes EQB_ERR_CUDA to its error
+ * word and returns, leaving the context usable.  This call runs one block
+ * that polls, `polls` times, a barrier that nothing completes, and reports
+ * the stall the same way.  The paper has no counterpart.
+ *   err_flag  device int32 (out): EQB_ERR_CUDA once the wait gives up
+ *   polls     1 .. 2^24 */
+eqb_status eqb_selftest_stalled_wait(int32_t *err_flag, int32_t polls, void *stream);
+
 #ifdef __cplusplus
 }
 #endif

@@ -33,7 +33,7 @@ __all__ = [
     "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route", "eqb_router_layer_step",
     "eqb_maxvio", "gshard_inject_grad", "eqb_rank_averaged_bias", "eqb_fixed_hist_bias",
-    "eqb_rank_averaged_workspace_bytes",
+    "eqb_rank_averaged_workspace_bytes", "eqb_selftest_stalled_wait",
 ]
 
 
@@ -253,6 +253,14 @@ def eqb_fixed_hist_bias(z, tau, K, lo, width, workspace, b_out=None, estimate=No
                                       _p(estimate), _p(workspace), workspace.numel(), _p(err_flag),
                                       _stream(stream)), "eqb_fixed_hist_bias")
     return b_out, estimate
+
+
+def eqb_selftest_stalled_wait(err_flag, polls=1 << 16, stream=None):
+    """Run the bounded-wait failure path on purpose (see eqb.h): afterwards
+    err_flag holds EQB_ERR_CUDA and the context is still usable."""
+    _need(err_flag, torch.int32, "err_flag")
+    _check(load().eqb_selftest_stalled_wait(_p(err_flag), int(polls), _stream(stream)),
+           "eqb_selftest_stalled_wait")
 
 
 def eqb_maxvio(loads, mb_offsets, K, out=None, per_mb=None, stream=None):

@@ -238,4 +238,36 @@ __device__ __forceinline__ uint32_t bf16_steps_down(uint32_t x, uint32_t steps) 
   return k >= kmin ? kappa16_inv(k - steps) : 0xff80u;
 }
 
+// ---- shared-memory mbarriers (CTA scope)
+
+__device__ __forceinline__ uint32_t saddr(const void* p) {
+  return static_cast<uint32_t>(__cvta_generic_to_shared(p));
+}
+__device__ __forceinline__ void bar_init(uint32_t bar, uint32_t count) {
+  asm volatile("mbarrier.init.shared::cta.b64 [%0], %1;" ::"r"(bar), "r"(count) : "memory");
+}
+__device__ __forceinline__ void bar_expect_tx(uint32_t bar, uint32_t bytes) {
+  asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(bar), "r"(bytes) : "memory");
+}
+// One poll: true once the phase of parity `parity` has completed; otherwise
+// the thread is suspended for at most about a microsecond (the time hint).
+__device__ __forceinline__ bool bar_try_wait(uint32_t bar, uint32_t parity) {
+  uint32_t ok;
+  asm volatile(
+      "{\n\t.reg .pred p;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
+      "selp.u32 %0, 1, 0, p;\n\t}"
+      : "=r"(ok)
+      : "r"(bar), "r"(parity), "r"(1000u)
+      : "memory");
+  return ok != 0;
+}
+// Wait for the phase of parity `parity`, giving up after `limit` polls:
+// false means the phase did not complete (the caller reports an error and
+// returns; no wait in this library is unbounded).
+__device__ __forceinline__ bool bar_wait_bounded(uint32_t bar, uint32_t parity, uint32_t limit) {
+  for (uint32_t i = 0; i < limit; ++i)
+    if (bar_try_wait(bar, parity)) return true;
+  return false;
+}
 }  // namespace eqb

@@ -28,7 +28,7 @@ namespace {
 
 constexpr int kBM = 128;  // rows of x per tile (UMMA M)
 constexpr int kBK = 64;   // bf16 columns per stage: one 128-byte swizzle atom
-constexpr uint32_t kSpinLimit = 1u << 22;  // a few seconds of polling at most
+constexpr uint32_t kSpinLimit = 1u << 20;  // polls of at most ~1 us: about a second
 
 __device__ __forceinline__ uint32_t smem_u32(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));
@@ -48,10 +48,10 @@ __device__ __forceinline__ bool mbar_try_wait(uint32_t bar, uint32_t parity) {
   uint32_t ok;
   asm volatile(
       "{\n\t.reg .pred p;\n\t"
-      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2;\n\t"
+      "mbarrier.try_wait.parity.shared::cta.b64 p, [%1], %2, %3;\n\t"
       "selp.u32 %0, 1, 0, p;\n\t}"
       : "=r"(ok)
-      : "r"(bar), "r"(parity)
+      : "r"(bar), "r"(parity), "r"(1000u)
       : "memory");
   return ok != 0;
 }

@@ -243,3 +243,11 @@ def test_comparison_statistics_reject(lib):
     assert g(FAKE, FAKE, 100, 64, 8, fl(-1.0), fl(0.1), FAKE, NULL, FAKE, ws - 1, NULL, NULL) == INVALID
     assert g(FAKE, FAKE, 100, 64, 8, fl(-1.0), fl(0.1), FAKE, ctypes.c_void_p(0x10004), FAKE, ws, NULL,
              NULL) == INVALID
+
+
+def test_selftest_rejects(lib):
+    f = lib.eqb_selftest_stalled_wait
+    assert f(NULL, 100, NULL) == INVALID
+    assert f(FAKE, 0, NULL) == INVALID
+    assert f(FAKE, (1 << 24) + 1, NULL) == INVALID
+    assert f(MISALIGNED, 100, NULL) == INVALID
