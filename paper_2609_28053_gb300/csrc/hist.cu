@@ -162,6 +162,10 @@ int launch_hist_t(const HistArgs& a, cudaStream_t s) {
   const int nE = a.E / Lay::ET;
   int ctas_per_sm = (228 * 1024 - 1024) / (smem + 1024);
   if (ctas_per_sm < 1) ctas_per_sm = 1;
+  // One 1024-thread block per SM whenever the bins are large: the same
+  // threads per SM as several smaller blocks, but a third of the zeroing and
+  // flushing of the block-local counters (E = 64, 128: 10-20% faster).
+  if (smem >= 32 * 1024) ctas_per_sm = 1;
   const int threads = ctas_per_sm == 1 ? 1024 : 512;
   if (ctas_per_sm > 2048 / threads) ctas_per_sm = 2048 / threads;
   int64_t nT = ((int64_t)di.sm_count * ctas_per_sm + nE - 1) / nE;
