@@ -538,6 +538,31 @@ def main():
     ms_per_step = ms / args.steps
     value = world * T / (ms_per_step / 1e3)
 
+    # The same step captured once as a CUDA graph and replayed (launch
+    # overheads removed); reported beside the stream timing, not instead.
+    graph = None
+    if one_call:
+        try:
+            cg = torch.cuda.CUDAGraph()
+            gs = torch.cuda.Stream()
+            gs.wait_stream(stream)
+            torch.cuda.synchronize()
+            with torch.cuda.graph(cg, stream=gs, capture_error_mode="relaxed"):
+                step.run_step(gs)
+            rs = torch.cuda.current_stream()  # replay() launches on the current stream
+            cg.replay()
+            torch.cuda.synchronize()
+            ga, gb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            ga.record(rs)
+            for _ in range(args.steps):
+                cg.replay()
+            gb.record(rs)
+            torch.cuda.synchronize()
+            graph = {"ms_per_step": ga.elapsed_time(gb) / args.steps, "steps": args.steps}
+            del cg
+        except Exception as exc:  # capture not possible: say why instead of a number
+            graph = {"error": f"{type(exc).__name__}: {exc}"[:200]}
+
     # Per-kernel durations: the same work issued kernel by kernel on one
     # stream, each launch bracketed by CUDA events, in its own timed loop.
     nk = len(step.names)
@@ -645,7 +670,7 @@ def main():
                 "kernels": kernels,
                 "kernels_sequential_ms": seq_ms,
                 "clocks": clk, "e2e": e2e, "cpu_baseline": cpu_base,
-                "elements_per_s": value * E, "extras": ext}
+                "elements_per_s": value * E, "cuda_graph": graph, "extras": ext}
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
