@@ -16,6 +16,33 @@ namespace eqb {
 
 constexpr unsigned kFull = 0xffffffffu;
 
+// Programmatic dependent launch.  The step's kernels are launched as
+// dependents of the previous kernel in the stream, so a kernel's launch and
+// its block-local set-up overlap the previous kernel's drain; each kernel
+// calls griddep_wait() before it touches global memory (it returns once the
+// previous grid has completed and its writes are visible; a no-op for a grid
+// not launched as a dependent).  No kernel triggers its successor early:
+// measured on the global step, early triggers cost 60 us, while the implicit
+// trigger at completion saves 17 us against plain launches.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+
+// Launch `kern` as a programmatic dependent of the previous work in `s`.
+template <typename... KArgs, typename... Args>
+inline cudaError_t launch_dependent(void (*kern)(KArgs...), dim3 grid, dim3 block, size_t smem,
+                                    cudaStream_t s, Args... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = grid;
+  cfg.blockDim = block;
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = s;
+  cudaLaunchAttribute attr;
+  attr.id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr.val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = &attr;
+  cfg.numAttrs = 1;
+  return cudaLaunchKernelEx(&cfg, kern, args...);
+}
+
 // bf16 in the low / high half of a packed word -> fp32 (exact).
 __device__ __forceinline__ float bf16_lo(uint32_t w) { return __uint_as_float(w << 16); }
 __device__ __forceinline__ float bf16_hi(uint32_t w) { return __uint_as_float(w & 0xffff0000u); }

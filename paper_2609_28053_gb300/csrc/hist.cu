@@ -70,6 +70,7 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
       sel[p] = (ue << 8) | (uo << 24);
     }
   };
+  griddep_wait();  // the bins were zeroed above; global reads start here
   if (PASS == 2 && !a.shard_off) load_sel(a.u);
   __syncthreads();
 
@@ -177,8 +178,7 @@ int launch_hist_t(const HistArgs& a, cudaStream_t s) {
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
     return kErrCuda;
   dim3 grid((unsigned)nE, (unsigned)nT);
-  kern<<<grid, threads, smem, s>>>(a, tpc);
-  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+  return launch_dependent(kern, grid, dim3(threads), smem, s, a, tpc) == cudaSuccess ? kOk : kErrCuda;
 }
 
 template <int PASS>

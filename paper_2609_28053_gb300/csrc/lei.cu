@@ -25,6 +25,7 @@ __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tok
   __shared__ __align__(16) float coef[kMaxE];
   __shared__ double red[kLeiThreads / 32];
   __shared__ double scal[2];
+  griddep_wait();
   const int E = a.E, E4 = a.E >> 2;
   const int64_t tb = (int64_t)blockIdx.x * tokens_per_cta;
   const int64_t te = min(tb + tokens_per_cta, a.T);
@@ -135,8 +136,9 @@ int launch_lei(const LeiArgs& a, cudaStream_t s) {
   if (grid > max_grid) grid = max_grid;
   if (grid < 1) grid = 1;
   const int64_t tpc = (a.T + grid - 1) / grid;
-  lei_kernel<<<(unsigned)grid, kLeiThreads, 0, s>>>(a, tpc);
-  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+  return launch_dependent(lei_kernel, dim3((unsigned)grid), dim3(kLeiThreads), 0, s, a, tpc) == cudaSuccess
+             ? kOk
+             : kErrCuda;
 }
 
 }  // namespace eqb

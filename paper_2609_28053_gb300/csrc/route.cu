@@ -64,6 +64,7 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
   uint16_t* ent = reinterpret_cast<uint16_t*>(wreg + nbuf * tile_bytes);
   int* wl = reinterpret_cast<int*>(wreg + nbuf * tile_bytes + nch * 32 * 2);
 
+  griddep_wait();
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
     const float v = a.b[e];
     bs[e] = v;
@@ -311,8 +312,9 @@ int launch_route_kp1(const RouteArgs& a, cudaStream_t s) {
   auto kern = route_kernel<KP1, G>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
     return kErrCuda;
-  kern<<<(unsigned)grid, nw * 32, smem, s>>>(a, tpw, nbuf);
-  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+  return launch_dependent(kern, dim3((unsigned)grid), dim3(nw * 32), smem, s, a, tpw, nbuf) == cudaSuccess
+             ? kOk
+             : kErrCuda;
 }
 
 }  // namespace

@@ -94,6 +94,7 @@ __global__ void __launch_bounds__(32 * wide_max_warps<E>(), 1)
   int* wl = reinterpret_cast<int*>(wreg + L::TILE + L::ENT);
   const uint32_t bar = saddr(wreg + L::TILE + L::ENT + L::WL);
 
+  griddep_wait();
   for (int e = threadIdx.x; e < E; e += blockDim.x) {
     const float v = a.b[e];
     bs[e] = v;
@@ -333,8 +334,8 @@ int launch_wide_t(const RouteArgs& a, cudaStream_t s) {
   auto kern = route_wide_kernel<E, KP1>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
     return kErrCuda;
-  kern<<<(unsigned)grid, nw * 32, smem, s>>>(a, tpw);
-  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+  return launch_dependent(kern, dim3((unsigned)grid), dim3(nw * 32), smem, s, a, tpw) == cudaSuccess ? kOk
+                                                                                         : kErrCuda;
 }
 
 template <int E>

@@ -24,6 +24,7 @@ __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__
                                                      int32_t* __restrict__ rho,
                                                      uint16_t* __restrict__ q_hat, int32_t* err,
                                                      const int64_t* __restrict__ shard_off, int K) {
+  griddep_wait();
   const int lane = threadIdx.x & 31;
   const int e = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (e >= E) return;
@@ -109,6 +110,7 @@ __device__ __forceinline__ void bf16_exp_range(uint32_t x, int& lo, int& hi) {
 // thread sums in ascending order.
 __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, float* __restrict__ b_next) {
   __shared__ double mean;
+  griddep_wait();
   if (threadIdx.x < 32) {
     const int lane = threadIdx.x;
     double part = 0.0;
@@ -151,21 +153,26 @@ __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, fl
 int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, int32_t* rho,
                   uint16_t* q_hat, int32_t* err, cudaStream_t s) {
   const int wpb = 8;
-  select_kernel<<<(E + wpb - 1) / wpb, wpb * 32, 0, s>>>(hist, E, pass, r, u, rho, q_hat, err, nullptr, 0);
-  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+  const int64_t* none = nullptr;
+  return launch_dependent(select_kernel, dim3((E + wpb - 1) / wpb), dim3(wpb * 32), 0, s, hist, E, pass, r, u, rho,
+                          q_hat, err, none, 0) == cudaSuccess
+             ? kOk
+             : kErrCuda;
 }
 
 int launch_select_sharded(const int32_t* hist, int E, int pass, const int64_t* shard_off, int P, int K,
                           uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err, cudaStream_t s) {
   const int wpb = 8;
   dim3 grid((E + wpb - 1) / wpb, P);
-  select_kernel<<<grid, wpb * 32, 0, s>>>(hist, E, pass, 0, u, rho, q_hat, err, shard_off, K);
-  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+  return launch_dependent(select_kernel, grid, dim3(wpb * 32), 0, s, hist, E, pass, (int64_t)0, u, rho, q_hat, err,
+                          shard_off, K) == cudaSuccess
+             ? kOk
+             : kErrCuda;
 }
 
 int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t s) {
-  bias_update_kernel<<<1, 256, 0, s>>>(q_hat, E, b_next);
-  return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
+  return launch_dependent(bias_update_kernel, dim3(1), dim3(256), 0, s, q_hat, E, b_next) == cudaSuccess ? kOk
+                                                                                                   : kErrCuda;
 }
 
 }  // namespace eqb
