@@ -143,9 +143,19 @@ class Step:
         self.r_global = None
         self.off_h = even_offsets(T, self.M)
         self.workspace = torch.zeros(eqb.eqb_layer_workspace_bytes(E), dtype=torch.uint8, device=dev)
-        self.names = (["router_route"] if workload == "router" else ["route_topk"]) + [
-            "margin_hist_pass1", "select_pass1", "margin_hist_pass2",
-            "select_pass2", "bias_update", "lei_inject_grad"]
+        # The one-call step streams LEI inside the two histogram passes when
+        # the [M,E] coefficient table fits its workspace (M * E <= 65,536);
+        # the per-kernel breakdown issues the same kernels through their own
+        # entry points.
+        self.fused = self.M * E <= 65536
+        self.coef = torch.empty((self.M, E), dtype=torch.float32, device=dev)
+        first = ["router_route"] if workload == "router" else ["route_topk"]
+        if self.fused:
+            self.names = first + ["lei_coefficients", "margin_hist_lei_pass1", "select_pass1",
+                                  "margin_hist_lei_pass2", "select_pass2", "bias_update"]
+        else:
+            self.names = first + ["margin_hist_pass1", "select_pass1", "margin_hist_pass2",
+                                  "select_pass2", "bias_update", "lei_inject_grad"]
 
     def run_step(self, stream):
         """One step through the one-call entry point eqb_layer_step: routing,
@@ -188,25 +198,40 @@ class Step:
         else:
             rec(0, lambda: eqb.eqb_route_topk(z, self.b, self.K, self.off, self.idx, self.tau,
                                               self.loads, None, ws.err, stream))
-        rec(1, lambda: eqb.eqb_margin_hist_pass1(z, self.tau, ws.hist_hi, ws.err, stream))
+        if self.fused:
+            th = self.T // 2
+            rec(1, lambda: eqb.lei_coefficients(self.loads, self.off, self.K, ETA, C_NORM, self.coef, stream))
+            rec(2, lambda: eqb.eqb_margin_hist_lei(z, self.tau, 1, ws.hist_hi, g, self.coef, self.off, 0, th,
+                                                   err_flag=ws.err, stream=stream))
+        else:
+            rec(1, lambda: eqb.eqb_margin_hist_pass1(z, self.tau, ws.hist_hi, ws.err, stream))
         if world > 1:
             torch.distributed.all_reduce(ws.hist_hi)
-        rec(2, lambda: eqb.eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream))
-        rec(3, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
+        k = 3 if self.fused else 2
+        rec(k, lambda: eqb.eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream))
+        if self.fused:
+            rec(4, lambda: eqb.eqb_margin_hist_lei(z, self.tau, 2, ws.hist_lo, g, self.coef, self.off, th,
+                                                   self.T, u=ws.u, stream=stream))
+        else:
+            rec(3, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
         if world > 1:
             torch.distributed.all_reduce(ws.hist_lo)
-        rec(4, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err,
+        k += 2
+        rec(k, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err,
                                                     stream))
-        rec(5, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
-        rec(6, lambda: eqb.lei_inject_grad(g, self.loads, self.off, self.K, ETA, C_NORM, stream))
+        rec(k + 1, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
+        if not self.fused:
+            rec(6, lambda: eqb.lei_inject_grad(g, self.loads, self.off, self.K, ETA, C_NORM, stream))
         if self.workload == "router":
             self.b.copy_(self.b_next)  # b^(q+1) routes step q+1
 
     def launches_per_step(self):
         """Kernels of this library launched by one timed step (memsets and
-        torch copies excluded): routing, two histogram passes, two
-        selections, the bias update and LEI (for the router workload the
-        routing kernel is the router projection with routing)."""
+        torch copies excluded): routing, the LEI coefficient table, two
+        histogram passes carrying the injection, two selections and the bias
+        update; without the table, LEI in its own launch instead (for the
+        router workload the routing kernel is the router projection with
+        routing)."""
         return 7
 
     def algorithmic_bytes(self):
@@ -215,10 +240,14 @@ class Step:
         (2TE) and tau (4T); LEI reads and writes grad (8TE); the router
         projection reads x (2Td) and W_r (2Ed) and writes z (2TE).  Per kernel:"""
         T, E, K = self.T, self.E, self.K
+        th = T // 2
         d = {"route_topk": 2 * T * E + 4 * T * K + 4 * T,
              "margin_hist_pass1": 2 * T * E + 4 * T,
              "margin_hist_pass2": 2 * T * E + 4 * T,
              "lei_inject_grad": 8 * T * E,
+             # the fused passes: the pass's z and tau plus its share of grad
+             "margin_hist_lei_pass1": 2 * T * E + 4 * T + 8 * th * E,
+             "margin_hist_lei_pass2": 2 * T * E + 4 * T + 8 * (T - th) * E,
              "path": 12 * T * E + 8 * T + 4 * T * K}
         if self.workload == "router":
             # the projection reads x and W_r and writes z; routing from its

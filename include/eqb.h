@@ -154,15 +154,49 @@ eqb_status lei_inject_grad(float *grad_s, const int32_t *loads,
                            const int64_t *mb_offsets, int32_t M, int64_t T,
                            int32_t E, int32_t K, float eta, float c, void *stream);
 
+/* The Load-Error Injection coefficients (Sec. 4, Eqs. LEI and norm) as a
+ * table: coef[l, e] = (float)(eta * sigma_l * rho_{l,e}), rho and sigma of
+ * microbatch l as in lei_inject_grad, by the same fp64 arithmetic (so the
+ * same bits as the coefficient lei_inject_grad adds).  An empty microbatch
+ * gets a row of zeros.
+ *   loads  device int32 [M,E]                          (in)
+ *   coef   device fp32 [M,E], 16-byte aligned          (out) */
+eqb_status lei_coefficients(const int32_t *loads, const int64_t *mb_offsets,
+                            int32_t M, int32_t E, int32_t K, float eta, float c,
+                            float *coef, void *stream);
+
+/* A histogram pass of Algorithm 1 with part of Load-Error Injection streamed
+ * beside it, in one kernel: pass 1 is eqb_margin_hist_pass1 (hist = hist_hi,
+ * err_flag used, u ignored), pass 2 is eqb_margin_hist_pass2 (hist =
+ * hist_lo, u required, err_flag ignored), and for the tokens t in
+ * [lei_t0, lei_t1) every grad_s[t, e] += coef[l(t), e] in fp32, l(t) the
+ * microbatch of t (Sec. 4, Eq. LEI).  The counting is issue-bound and the
+ * injection DRAM-bound, so the two share the GPU better than back to back.
+ * Results are bit-identical to the separate calls; the one-call step runs
+ * pass 1 with the first half of the tokens and pass 2 with the rest.
+ *   grad_s  device fp32 [T,E], 16-byte aligned, updated in place on [lei_t0, lei_t1)
+ *   coef    device fp32 [M,E] from lei_coefficients, 16-byte aligned
+ *   0 <= lei_t0 <= lei_t1 <= T, else EQB_ERR_INVALID_ARG. */
+eqb_status eqb_margin_hist_lei(const eqb_bf16 *z, const float *tau, int64_t T,
+                               int32_t E, int32_t pass, const uint8_t *u,
+                               int32_t *hist, int32_t *err_flag, float *grad_s,
+                               const float *coef, const int64_t *mb_offsets,
+                               int32_t M, int64_t lei_t0, int64_t lei_t1,
+                               void *stream);
+
 /* Bytes of device workspace eqb_layer_step needs for E experts (the two
- * [E,256] histograms, u, rho and q_hat, each 256-byte aligned). */
+ * [E,256] histograms, u, rho, q_hat and a 65,536-float LEI coefficient
+ * table, each 256-byte aligned). */
 size_t eqb_layer_workspace_bytes(int32_t E);
 
 /* One layer's whole routing-balance step in one call, in the paper's order:
  * routing (Sec. 2), Algorithm 1's coarse pass, selection, fine pass,
  * selection, the Eq. (2) bias update, then Load-Error Injection (Sec. 4,
  * Eqs. LEI and norm) on grad_s when grad_s is given.  Results are identical
- * to the individual calls above.
+ * to the individual calls above.  When M * E <= 65,536 the LEI coefficients
+ * are formed right after routing (lei_coefficients) and the injection is
+ * streamed by the two histogram passes, half of the tokens each
+ * (eqb_margin_hist_lei); otherwise LEI runs last (lei_inject_grad).
  *   z, b, mb_offsets, M, topk_idx (nullable), tau, eta, c: as in
  *             eqb_route_topk / lei_inject_grad;
  *   mb_offsets_host host copy of mb_offsets (nullable; validated when given)

@@ -33,7 +33,8 @@ __all__ = [
     "EqbWorkspace", "eqb_layer_forward", "eqb_router_logits", "eqb_layer_workspace_bytes",
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route", "eqb_router_layer_step",
     "eqb_maxvio", "gshard_inject_grad", "eqb_rank_averaged_bias", "eqb_fixed_hist_bias",
-    "eqb_rank_averaged_workspace_bytes", "eqb_selftest_stalled_wait",
+    "eqb_rank_averaged_workspace_bytes", "eqb_selftest_stalled_wait", "lei_coefficients",
+    "eqb_margin_hist_lei",
 ]
 
 
@@ -142,6 +143,39 @@ def lei_inject_grad(grad_s, loads, mb_offsets, K, eta, c, stream=None):
     _need(loads, torch.int32, "loads", (M, E))
     _check(load().lei_inject_grad(_p(grad_s), _p(loads), _p(mb_offsets), M, T, E, K, float(eta),
                                   float(c), _stream(stream)), "lei_inject_grad")
+
+
+def lei_coefficients(loads, mb_offsets, K, eta, c, coef=None, stream=None):
+    """The [M,E] table of LEI coefficients eta * sigma_l * rho_{l,e} (the
+    values lei_inject_grad adds).  Returns coef (fp32 [M,E])."""
+    M, E = loads.shape
+    _need(loads, torch.int32, "loads")
+    _need(mb_offsets, torch.int64, "mb_offsets", (M + 1,))
+    if coef is None:
+        coef = torch.empty((M, E), dtype=torch.float32, device=loads.device)
+    _need(coef, torch.float32, "coef", (M, E))
+    _check(load().lei_coefficients(_p(loads), _p(mb_offsets), M, E, int(K), float(eta), float(c), _p(coef),
+                                   _stream(stream)), "lei_coefficients")
+    return coef
+
+
+def eqb_margin_hist_lei(z, tau, pass_, hist, grad_s, coef, mb_offsets, lei_t0, lei_t1, u=None,
+                        err_flag=None, stream=None):
+    """A histogram pass (1: coarse, 2: fine, needs u) with grad_s[t] +=
+    coef[mb(t)] for t in [lei_t0, lei_t1) streamed beside it, one kernel."""
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(tau, torch.float32, "tau", (T,))
+    _need(hist, torch.int32, "hist", (E, 256))
+    _need(u, torch.uint8, "u", (E,))
+    _need(err_flag, torch.int32, "err_flag")
+    _need(grad_s, torch.float32, "grad_s", (T, E))
+    _need(mb_offsets, torch.int64, "mb_offsets")
+    M = mb_offsets.numel() - 1
+    _need(coef, torch.float32, "coef", (M, E))
+    _check(load().eqb_margin_hist_lei(_p(z), _p(tau), T, E, int(pass_), _p(u), _p(hist), _p(err_flag),
+                                      _p(grad_s), _p(coef), _p(mb_offsets), M, int(lei_t0), int(lei_t1),
+                                      _stream(stream)), "eqb_margin_hist_lei")
 
 
 def eqb_router_logits(x, W_r, z=None, err_flag=None, stream=None):

@@ -155,6 +155,36 @@ eqb_status lei_inject_grad(float* grad_s, const int32_t* loads, const int64_t* m
   return to_status(eqb::launch_lei(a, as_stream(stream)));
 }
 
+eqb_status lei_coefficients(const int32_t* loads, const int64_t* mb_offsets, int32_t M, int32_t E, int32_t K,
+                            float eta, float c, float* coef, void* stream) {
+  eqb_status st = check_shape(0, E, K, true);
+  if (st != EQB_OK) return st;
+  if (!loads || !mb_offsets || !coef || M < 1) return EQB_ERR_INVALID_ARG;
+  if (!(eta == eta) || !(c == c)) return EQB_ERR_INVALID_ARG;
+  if (!aligned(loads, 4) || !aligned(mb_offsets, 8) || !aligned(coef, 16)) return EQB_ERR_INVALID_ARG;
+  eqb::LeiArgs a{nullptr, loads, mb_offsets, M, 0, 0, E, K, eta, c};
+  return to_status(eqb::launch_lei_coef(a, coef, as_stream(stream)));
+}
+
+eqb_status eqb_margin_hist_lei(const eqb_bf16* z, const float* tau, int64_t T, int32_t E, int32_t pass,
+                               const uint8_t* u, int32_t* hist, int32_t* err_flag, float* grad_s,
+                               const float* coef, const int64_t* mb_offsets, int32_t M, int64_t lei_t0,
+                               int64_t lei_t1, void* stream) {
+  eqb_status st = check_shape(T, E, 1, false);
+  if (st != EQB_OK) return st;
+  if (pass != 1 && pass != 2) return EQB_ERR_INVALID_ARG;
+  if (!z || !tau || !hist || (pass == 2 && !u) || !grad_s || !coef || !mb_offsets || M < 1)
+    return EQB_ERR_INVALID_ARG;
+  if (lei_t0 < 0 || lei_t1 < lei_t0 || lei_t1 > T) return EQB_ERR_INVALID_ARG;
+  if (!aligned(z, 16) || !aligned(tau, 4) || !aligned(hist, 4) || !aligned(err_flag, 4) ||
+      !aligned(grad_s, 16) || !aligned(coef, 16) || !aligned(mb_offsets, 8))
+    return EQB_ERR_INVALID_ARG;
+  if (T == 0) return EQB_OK;
+  eqb::HistArgs h{z, tau, T, E, pass == 2 ? u : nullptr, hist, pass == 1 ? err_flag : nullptr};
+  eqb::LeiStream ls{grad_s, coef, mb_offsets, M, lei_t0, lei_t1};
+  return to_status(eqb::launch_hist_lei(h, pass, ls, as_stream(stream)));
+}
+
 eqb_status eqb_router_logits(const eqb_bf16* x, const eqb_bf16* W_r, int64_t T, int32_t d, int32_t E,
                              eqb_bf16* z, int32_t* err_flag, void* stream) {
   if (T < 0 || d < 1 || E < 1) return EQB_ERR_INVALID_ARG;

@@ -69,6 +69,17 @@ struct LeiArgs {
   float eta, c;
 };
 
+// Load-Error Injection streamed by a histogram pass beside its own work:
+// grad_s[t, e] += coef[mb(t), e] for the tokens [t0, t1), from the [M,E]
+// coefficient table of launch_lei_coef.  Token numbers are absolute.
+struct LeiStream {
+  float* g = nullptr;  // nullptr: no injection
+  const float* coef = nullptr;
+  const int64_t* off = nullptr;
+  int M = 0;
+  int64_t t0 = 0, t1 = 0;
+};
+
 struct GshardArgs {
   float* g;
   const uint16_t* z;
@@ -80,14 +91,20 @@ struct GshardArgs {
   float alpha;
 };
 
+// Capacity (floats) of the step's LEI coefficient table: the fused step
+// (injection streamed by the histogram passes) runs when M * E fits.
+constexpr int64_t kLeiCoefCap = 65536;
+
 // The step's scratch, carved from one caller-provided buffer (256-byte
-// aligned pieces): the two [E,256] histograms, u, rho and q_hat.
+// aligned pieces): the two [E,256] histograms, u, rho, q_hat and the
+// [M,E] LEI coefficient table.
 struct StepWorkspace {
   int32_t* H;
   int32_t* L;
   uint8_t* u;
   int32_t* rho;
   uint16_t* q;
+  float* coef;
 };
 // Carves `base` (or, with base == nullptr, only measures); returns the bytes used.
 size_t carve_workspace(void* base, int E, StepWorkspace* w);
@@ -96,6 +113,8 @@ int launch_route(const RouteArgs& a, cudaStream_t s);
 bool route_wide_supported(int E, int K);
 int launch_route_wide(const RouteArgs& a, cudaStream_t s);
 int launch_hist(const HistArgs& a, int pass, cudaStream_t s);
+// A histogram pass (1 or 2) with the injection `ls` streamed beside it.
+int launch_hist_lei(const HistArgs& a, int pass, const LeiStream& ls, cudaStream_t s);
 int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, int32_t* rho,
                   uint16_t* q_hat, int32_t* err, cudaStream_t s);
 // One selection per token shard (device int64 [P+1]): shard p reads
@@ -105,6 +124,9 @@ int launch_select_sharded(const int32_t* hist, int E, int pass, const int64_t* s
                           uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err, cudaStream_t s);
 int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t s);
 int launch_lei(const LeiArgs& a, cudaStream_t s);
+// The [M,E] fp32 table of Eq. (norm) coefficients, row l for microbatch l
+// (bit-identical to the coefficients launch_lei forms).
+int launch_lei_coef(const LeiArgs& a, float* coef, cudaStream_t s);
 int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, uint16_t* z,
                        int32_t* err, cudaStream_t s);
 int launch_gshard(const GshardArgs& a, cudaStream_t s);

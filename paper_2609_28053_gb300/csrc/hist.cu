@@ -26,6 +26,16 @@
 // tokens; the flush is also how token partitions are summed in device memory.
 // Each lane keeps eight 16-byte loads in flight (eight tokens per round),
 // which covers the DRAM latency without L2 prefetches.
+//
+// Fused with Load-Error Injection (the one-call step): the passes are bound
+// by issue, not by DRAM, while LEI (Sec. 4) is a pure DRAM stream that needs
+// only the loads.  A fused block gives a quarter of its warps to streaming
+// grad_s[t, e] += coef[mb(t), e] over its slice of a token range from the
+// start, the other warps count, and each counting warp joins the stream when
+// its counting is done; the stream is cut into chunks of about 8 KiB of
+// grad_s handed out by a shared counter, so no warp idles while the block
+// has work.  Each pass carries half of the step's tokens, which turns both
+// passes into DRAM-bound ones.
 #include "eqb_device.cuh"
 
 namespace eqb {
@@ -34,6 +44,82 @@ namespace {
 
 constexpr int kUnroll = 8;  // 16-byte loads in flight per lane (64 registers at 1024 threads)
 constexpr int64_t kFlushTokens = 65535;
+constexpr int kLeiUnroll = 8;  // 16-byte grad_s loads in flight per lane in the injection stream
+
+// The injection share of a fused block (see above): chunks of about 8 KiB of
+// grad_s from this block's slice of [ls.t0, ls.t1), taken through the shared
+// counter *next.  Every element gets one fp32 addition (round to nearest) of
+// its microbatch's coefficient, as in lei.cu.
+__device__ __forceinline__ void stream_lei(const LeiStream& ls, int E, int* next) {
+  const int lane = threadIdx.x & 31;
+  const int64_t nct = (int64_t)gridDim.x * gridDim.y;
+  const int64_t cta = (int64_t)blockIdx.y * gridDim.x + blockIdx.x;
+  const int64_t n = ls.t1 - ls.t0;
+  const int64_t per = (n + nct - 1) / nct;
+  const int64_t q0 = ls.t0 + min(cta * per, n);
+  const int64_t q1 = ls.t0 + min(cta * per + per, n);
+  const int E4 = E >> 2;
+  const int ch = max(1, 512 / E4);  // tokens per chunk
+  const int dcol = 32 % E4;
+  float4* g4 = reinterpret_cast<float4*>(ls.g);
+  const float4* c4 = reinterpret_cast<const float4*>(ls.coef);
+  int64_t mlo = 1, mhi = 0;  // token range of microbatch ml (none yet)
+  int ml = 0;
+  for (;;) {
+    int c = 0;
+    if (lane == 0) c = atomicAdd(next, 1);
+    c = __shfl_sync(kFull, c, 0);
+    int64_t ta = q0 + (int64_t)c * ch;
+    if (ta >= q1) break;
+    const int64_t tb = min(ta + ch, q1);
+    while (ta < tb) {
+      if (ta < mlo || ta >= mhi) {
+        ml = microbatch_of(ls.off, ls.M, ta);
+        mlo = __ldg(ls.off + ml);
+        mhi = __ldg(ls.off + ml + 1);
+      }
+      // Malformed offsets (off[M] < T): tokens past the last boundary are
+      // the last microbatch's, as in lei.cu.
+      const int64_t se = mhi > ta ? min(tb, mhi) : tb;
+      const float4* crow = c4 + (int64_t)ml * E4;
+      int64_t i = ta * E4 + lane;
+      const int64_t i1 = se * E4;
+      int col = static_cast<int>(i % E4);
+      for (; i + 32 * (kLeiUnroll - 1) < i1; i += 32 * kLeiUnroll) {
+        float4 v[kLeiUnroll];
+        int cc[kLeiUnroll];
+#pragma unroll
+        for (int u = 0; u < kLeiUnroll; ++u) {
+          v[u] = __ldcs(g4 + i + 32 * u);
+          cc[u] = col;
+          col += dcol;
+          if (col >= E4) col -= E4;
+        }
+#pragma unroll
+        for (int u = 0; u < kLeiUnroll; ++u) {
+          const float4 cf = __ldg(crow + cc[u]);
+          v[u].x = __fadd_rn(v[u].x, cf.x);
+          v[u].y = __fadd_rn(v[u].y, cf.y);
+          v[u].z = __fadd_rn(v[u].z, cf.z);
+          v[u].w = __fadd_rn(v[u].w, cf.w);
+          __stcs(g4 + i + 32 * u, v[u]);
+        }
+      }
+      for (; i < i1; i += 32) {
+        float4 v = __ldcs(g4 + i);
+        const float4 cf = __ldg(crow + col);
+        v.x = __fadd_rn(v.x, cf.x);
+        v.y = __fadd_rn(v.y, cf.y);
+        v.z = __fadd_rn(v.z, cf.z);
+        v.w = __fadd_rn(v.w, cf.w);
+        __stcs(g4 + i, v);
+        col += dcol;
+        if (col >= E4) col -= E4;
+      }
+      ta = se;
+    }
+  }
+}
 
 template <int LPT>
 struct HistLayout {
@@ -44,18 +130,26 @@ struct HistLayout {
   __host__ __device__ static int row_word(int row) { return row * 256 + (row >> 2); }
 };
 
-template <int PASS, int LPT>
-__global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_per_cta) {
+template <int PASS, int LPT, bool LEI>
+__global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_per_cta, LeiStream ls) {
   using Lay = HistLayout<LPT>;
   extern __shared__ __align__(16) uint32_t bins[];
+  __shared__ int lei_next;  // next injection chunk of this block (fused only)
   const int E = a.E;
   const int e0 = blockIdx.x * Lay::ET;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
-  const int nw = blockDim.x >> 5;
+  const int nw = LEI ? (blockDim.x >> 5) - (blockDim.x >> 7) : (blockDim.x >> 5);  // counting warps
+  const int nt = nw * 32;
   const int c = lane % LPT;     // 8-expert chunk of the tile owned by this lane
   const int tok = lane / LPT;   // token slot inside the warp step
+  // Barrier of the counting warps (all warps unless fused).
+  auto sync_counting = [&]() {
+    if (LEI) asm volatile("bar.sync 1, %0;" ::"r"(nt) : "memory");
+    else __syncthreads();
+  };
 
   for (int i = threadIdx.x; i < Lay::kWords; i += blockDim.x) bins[i] = 0u;
+  if (LEI && threadIdx.x == 0) lei_next = 0;
   // Shared address of this lane's first pair row; pair p adds p * 1 KiB.
   const uint32_t base = static_cast<uint32_t>(__cvta_generic_to_shared(bins)) +
                         4u * static_cast<uint32_t>(Lay::row_word(4 * c));
@@ -73,6 +167,10 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
   griddep_wait();  // the bins were zeroed above; global reads start here
   if (PASS == 2 && !a.shard_off) load_sel(a.u);
   __syncthreads();
+  if (LEI && wid >= nw) {
+    stream_lei(ls, E, &lei_next);
+    return;
+  }
 
   // Token indices fit in 32 bits (T < 2^31 is checked on the host).
   const int tb = static_cast<int>(min((int64_t)blockIdx.y * tokens_per_cta, a.T));
@@ -134,9 +232,9 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
       for (int u = 0; u < kUnroll; ++u) process(w[u], tt[u]);
     }
     for (; t < ce; t += step, zp += zstride) process(__ldcs(reinterpret_cast<const uint4*>(zp)), __ldg(a.tau + t));
-    __syncthreads();
+    sync_counting();
     // Flush: add every non-zero 16-bit counter to the global histogram.
-    for (int i = threadIdx.x; i < Lay::kRows * 256; i += blockDim.x) {
+    for (int i = threadIdx.x; i < Lay::kRows * 256; i += nt) {
       const int row = i >> 8, slot = i & 255;
       const int wi = Lay::row_word(row) + slot;
       const uint32_t v = bins[wi];
@@ -149,13 +247,14 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
         if (PASS == 1 && (bin == 0 || bin == 255)) raise_flag(a.err, kErrNonfinite);
       }
     }
-    __syncthreads();
+    sync_counting();
     cb = ce;
   }
+  if (LEI) stream_lei(ls, E, &lei_next);
 }
 
-template <int PASS, int LPT>
-int launch_hist_t(const HistArgs& a, cudaStream_t s) {
+template <int PASS, int LPT, bool LEI>
+int launch_hist_t(const HistArgs& a, const LeiStream& ls, cudaStream_t s) {
   using Lay = HistLayout<LPT>;
   DeviceInfo di;
   if (int rc = device_info(&di)) return rc;
@@ -174,28 +273,34 @@ int launch_hist_t(const HistArgs& a, cudaStream_t s) {
   if (nT > max_nT) nT = max_nT;
   if (nT < 1) nT = 1;
   const int64_t tpc = (a.T + nT - 1) / nT;
-  auto kern = hist_kernel<PASS, LPT>;
+  auto kern = hist_kernel<PASS, LPT, LEI>;
   if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) != cudaSuccess)
     return kErrCuda;
   dim3 grid((unsigned)nE, (unsigned)nT);
-  return launch_dependent(kern, grid, dim3(threads), smem, s, a, tpc) == cudaSuccess ? kOk : kErrCuda;
+  return launch_dependent(kern, grid, dim3(threads), smem, s, a, tpc, ls) == cudaSuccess ? kOk : kErrCuda;
 }
 
-template <int PASS>
-int launch_hist_pass(const HistArgs& a, cudaStream_t s) {
-  if (a.E % 256 == 0) return launch_hist_t<PASS, 32>(a, s);
-  if (a.E % 128 == 0) return launch_hist_t<PASS, 16>(a, s);
-  if (a.E % 64 == 0) return launch_hist_t<PASS, 8>(a, s);
-  if (a.E % 32 == 0) return launch_hist_t<PASS, 4>(a, s);
-  if (a.E % 16 == 0) return launch_hist_t<PASS, 2>(a, s);
-  return launch_hist_t<PASS, 1>(a, s);
+template <int PASS, bool LEI>
+int launch_hist_pass(const HistArgs& a, const LeiStream& ls, cudaStream_t s) {
+  if (a.E % 256 == 0) return launch_hist_t<PASS, 32, LEI>(a, ls, s);
+  if (a.E % 128 == 0) return launch_hist_t<PASS, 16, LEI>(a, ls, s);
+  if (a.E % 64 == 0) return launch_hist_t<PASS, 8, LEI>(a, ls, s);
+  if (a.E % 32 == 0) return launch_hist_t<PASS, 4, LEI>(a, ls, s);
+  if (a.E % 16 == 0) return launch_hist_t<PASS, 2, LEI>(a, ls, s);
+  return launch_hist_t<PASS, 1, LEI>(a, ls, s);
 }
 
 }  // namespace
 
 int launch_hist(const HistArgs& a, int pass, cudaStream_t s) {
-  if (pass == 3) return launch_hist_pass<3>(a, s);
-  return pass == 1 ? launch_hist_pass<1>(a, s) : launch_hist_pass<2>(a, s);
+  const LeiStream none;
+  if (pass == 3) return launch_hist_pass<3, false>(a, none, s);
+  return pass == 1 ? launch_hist_pass<1, false>(a, none, s) : launch_hist_pass<2, false>(a, none, s);
+}
+
+int launch_hist_lei(const HistArgs& a, int pass, const LeiStream& ls, cudaStream_t s) {
+  if (!ls.g || !ls.coef || !ls.off || ls.M < 1 || ls.t0 < 0 || ls.t1 < ls.t0) return kErrInvalidArg;
+  return pass == 1 ? launch_hist_pass<1, true>(a, ls, s) : launch_hist_pass<2, true>(a, ls, s);
 }
 
 }  // namespace eqb

@@ -12,6 +12,10 @@
 // microbatch it meets (fp64, the threads striding over the experts, a block
 // max for xi) into shared memory as fp32, and then streams its range with
 // 16-byte loads and stores using evict-first cache hints.
+//
+// For the one-call step the coefficients are also formed once per microbatch
+// into an [M,E] table (lei_coef_kernel), from which the histogram passes
+// stream the injection beside their own work (hist.cu).
 #include "eqb_device.cuh"
 
 namespace eqb {
@@ -21,10 +25,56 @@ namespace {
 constexpr int kLeiThreads = 256;
 constexpr int kLeiUnroll = 4;
 
-__global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tokens_per_cta) {
-  __shared__ __align__(16) float coef[kMaxE];
+// Eq. (norm) coefficients eta * sigma * rho_e of one microbatch with n tokens
+// and loads f (one row of [M,E]), computed by a whole block of kLeiThreads
+// threads into out[0..E) (shared or global memory) and visible to the block
+// on return.  fp64 throughput is low on this part, so each thread does only
+// a multiply-add and a multiply per expert; the reciprocal of the target
+// load and tanh are formed once.
+__device__ void block_lei_coef(const int32_t* __restrict__ f, int64_t n, int E, int K, float eta, float c,
+                               float* out) {
   __shared__ double red[kLeiThreads / 32];
   __shared__ double scal[2];
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
+  __syncthreads();  // a previous call has finished reading scal and out
+  if (threadIdx.x == 0) scal[0] = n > 0 ? (double)E / ((double)K * (double)n) : 0.0;  // 1 / fbar
+  __syncthreads();
+  const double inv_fbar = scal[0];
+  // each thread holds the rho of experts threadIdx.x + k * kLeiThreads
+  constexpr int kPer = kMaxE / kLeiThreads;
+  double rho[kPer];
+  double amax = 0.0;
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int e = threadIdx.x + k * kLeiThreads;
+    rho[k] = (e < E && inv_fbar > 0.0) ? (double)__ldg(f + e) * inv_fbar - 1.0 : 0.0;
+    amax = fmax(amax, fabs(rho[k]));
+  }
+#pragma unroll
+  for (int d = 16; d > 0; d >>= 1) amax = fmax(amax, __shfl_xor_sync(kFull, amax, d));
+  if (lane == 0) red[wid] = amax;
+  __syncthreads();
+  if (threadIdx.x == 0) {
+    double rmax = red[0];
+    for (int w = 1; w < kLeiThreads / 32; ++w) rmax = fmax(rmax, red[w]);
+    double sigma = 1.0;
+    if (c > 0.0f) {
+      const double xi = rmax / (double)c;
+      sigma = (xi == 0.0) ? 1.0 : tanh(xi) / xi;
+    }
+    scal[1] = (double)eta * sigma;
+  }
+  __syncthreads();
+#pragma unroll
+  for (int k = 0; k < kPer; ++k) {
+    const int e = threadIdx.x + k * kLeiThreads;
+    if (e < E) out[e] = __double2float_rn(scal[1] * rho[k]);
+  }
+  __syncthreads();
+}
+
+__global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tokens_per_cta) {
+  __shared__ __align__(16) float coef[kMaxE];
   griddep_wait();
   const int E = a.E, E4 = a.E >> 2;
   const int64_t tb = (int64_t)blockIdx.x * tokens_per_cta;
@@ -32,7 +82,6 @@ __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tok
   if (tb >= te) return;
   float4* g4 = reinterpret_cast<float4*>(a.g);
   const float4* c4 = reinterpret_cast<const float4*>(coef);
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
 
   int64_t t = tb;
   while (t < te) {
@@ -41,48 +90,7 @@ __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tok
     // Malformed offsets (off[M] < T) must not stall the loop: tokens past
     // the last boundary are treated as the last microbatch's.
     const int64_t seg_end = (hi > t) ? min(te, hi) : te;
-
-    // ---- coefficients of microbatch l.  fp64 throughput is low on this
-    // part, so each thread does only a multiply-add and a multiply; the
-    // reciprocal of the target load and tanh are formed once per block.
-    __syncthreads();  // previous segment finished reading coef and scal
-    if (threadIdx.x == 0) {
-      const double n = (double)(hi - lo);
-      scal[0] = n > 0.0 ? (double)E / ((double)a.K * n) : 0.0;  // 1 / fbar
-    }
-    __syncthreads();
-    const double inv_fbar = scal[0];
-    // each thread holds the rho of experts threadIdx.x + k * blockDim.x
-    constexpr int kPer = kMaxE / kLeiThreads;
-    double rho[kPer];
-    double amax = 0.0;
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const int e = threadIdx.x + k * kLeiThreads;
-      rho[k] = (e < E && inv_fbar > 0.0) ? (double)__ldg(a.loads + (int64_t)l * E + e) * inv_fbar - 1.0 : 0.0;
-      amax = fmax(amax, fabs(rho[k]));
-    }
-#pragma unroll
-    for (int d = 16; d > 0; d >>= 1) amax = fmax(amax, __shfl_xor_sync(kFull, amax, d));
-    if (lane == 0) red[wid] = amax;
-    __syncthreads();
-    if (threadIdx.x == 0) {
-      double rmax = red[0];
-      for (int w = 1; w < (int)(blockDim.x >> 5); ++w) rmax = fmax(rmax, red[w]);
-      double sigma = 1.0;
-      if (a.c > 0.0f) {
-        const double xi = rmax / (double)a.c;
-        sigma = (xi == 0.0) ? 1.0 : tanh(xi) / xi;
-      }
-      scal[1] = (double)a.eta * sigma;
-    }
-    __syncthreads();
-#pragma unroll
-    for (int k = 0; k < kPer; ++k) {
-      const int e = threadIdx.x + k * kLeiThreads;
-      if (e < E) coef[e] = __double2float_rn(scal[1] * rho[k]);
-    }
-    __syncthreads();
+    block_lei_coef(a.loads + (int64_t)l * E, hi - lo, E, a.K, a.eta, a.c, coef);
 
     // ---- stream grad_s[t .. seg_end) in float4 units
     const int64_t i0 = t * E4, i1 = seg_end * E4;
@@ -125,7 +133,23 @@ __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tok
   }
 }
 
+// One block per microbatch: row l of the [M,E] coefficient table.
+__global__ void __launch_bounds__(kLeiThreads) lei_coef_kernel(LeiArgs a, float* coef) {
+  griddep_wait();
+  const int l = blockIdx.x;
+  const int64_t n = __ldg(a.off + l + 1) - __ldg(a.off + l);
+  block_lei_coef(a.loads + (int64_t)l * a.E, n, a.E, a.K, a.eta, a.c, coef + (int64_t)l * a.E);
+}
+
 }  // namespace
+
+int launch_lei_coef(const LeiArgs& a, float* coef, cudaStream_t s) {
+  if (a.M < 1) return kErrInvalidArg;
+  return launch_dependent(lei_coef_kernel, dim3((unsigned)a.M), dim3(kLeiThreads), 0, s, a, coef) ==
+                 cudaSuccess
+             ? kOk
+             : kErrCuda;
+}
 
 int launch_lei(const LeiArgs& a, cudaStream_t s) {
   DeviceInfo di;

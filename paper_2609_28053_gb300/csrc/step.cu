@@ -26,6 +26,7 @@ size_t carve_workspace(void* base, int E, StepWorkspace* w) {
   w->u = take(static_cast<size_t>(E));
   w->rho = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 4));
   w->q = reinterpret_cast<uint16_t*>(take(static_cast<size_t>(E) * 2));
+  w->coef = reinterpret_cast<float*>(take(static_cast<size_t>(kLeiCoefCap) * 4));
   return off;
 }
 
@@ -89,12 +90,30 @@ eqb_status clear(const Workspace& w, int32_t* loads, int32_t E, int32_t M, cudaS
 }
 
 // Everything after routing: Algorithm 1's two passes with their selections,
-// the Eq. (2) bias update and LEI.
+// the Eq. (2) bias update and LEI.  When the [M,E] coefficient table fits the
+// workspace, the coefficients are formed once and each histogram pass
+// streams the injection of half of the tokens beside its counting (the
+// passes are issue-bound, the injection DRAM-bound); the results are the
+// same bits as the separate LEI launch.
 eqb_status after_routing(const Workspace& w, const eqb_bf16* z, int64_t T, int32_t E, int32_t K,
                          const int64_t* mb_offsets, int32_t M, int64_t r, const float* tau,
                          const int32_t* loads, float* b_next, float* grad_s, float eta, float c,
                          int32_t* err_flag, cudaStream_t s) {
   eqb::HistArgs h1{z, tau, T, E, nullptr, w.H, err_flag};
+  if (grad_s && static_cast<int64_t>(M) * E <= eqb::kLeiCoefCap) {
+    eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
+    if (int rc = eqb::launch_lei_coef(la, w.coef, s)) return st(rc);
+    const int64_t th = T / 2;
+    eqb::LeiStream l1{grad_s, w.coef, mb_offsets, M, 0, th};
+    eqb::LeiStream l2{grad_s, w.coef, mb_offsets, M, th, T};
+    if (int rc = eqb::launch_hist_lei(h1, 1, l1, s)) return st(rc);
+    if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
+    eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};
+    if (int rc = eqb::launch_hist_lei(h2, 2, l2, s)) return st(rc);
+    if (int rc = eqb::launch_select(w.L, E, 2, r, w.u, w.rho, w.q, err_flag, s)) return st(rc);
+    if (int rc = eqb::launch_bias_update(w.q, E, b_next, s)) return st(rc);
+    return EQB_OK;
+  }
   if (int rc = eqb::launch_hist(h1, 1, s)) return st(rc);
   if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
   eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};

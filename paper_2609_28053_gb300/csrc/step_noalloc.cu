@@ -9,7 +9,7 @@
 // [E,256] histograms, u, rho and q_hat) lives here.
 //
 // The scratch is one file-scope device array sized for the largest supported
-// E (256 experts).  Every GPU that loads this library holds it (about 514
+// E (256 experts).  Every GPU that loads this library holds it (about 770
 // KiB) until the process exits.  Host code cannot use the array's name as a
 // device address, so the first call on each device, with that device
 // current, looks the address up once with cudaGetSymbolAddress; make that
@@ -26,7 +26,7 @@
 
 namespace {
 
-constexpr size_t kStaticWorkspaceBytes = 526080;  // eqb_layer_workspace_bytes(256)
+constexpr size_t kStaticWorkspaceBytes = 788224;  // eqb_layer_workspace_bytes(256)
 static __device__ __align__(256) unsigned char g_step_scratch[kStaticWorkspaceBytes];
 
 constexpr int kMaxDevices = 64;
