@@ -18,7 +18,7 @@
 //      filter threshold.
 //   B. per-chunk masks of U_e = bf16(z_e + RU(b_e)) >= threshold, every one
 //      of the experts with s_e >= tau_t among them, kept in shared memory,
-//      with a 32-bit set of the chunks that have a hit.
+//      with the set of non-zero mask words (32 experts each).
 //   C. the listed experts, in ascending index, are inserted into a sorted
 //      (K+1)-list by their exact fp32 score s_e = fp32(z_e) + b_e; a new
 //      element goes after equal scores, so ties keep the lower index first.
@@ -200,8 +200,8 @@ __global__ void __launch_bounds__(32 * wide_max_warps<E>(), 1)
     const uint32_t thf = bf16_steps_down(__float_as_uint(theta) >> 16, 4u);
     const uint32_t thf2 = thf | (thf << 16);
 
-    // ---- B: per-chunk masks of U >= threshold, stored four to a word, and
-    // the set of chunks with a hit as one bit per chunk
+    // ---- B: per-chunk masks of U >= threshold, stored four to a word (bit
+    // 8u + j of word k is expert 32k + 8u + j), and the set of non-zero words
     uint32_t hits = 0u;
 #pragma unroll
     for (int k = 0; k < NCH / 4; ++k) {
@@ -220,31 +220,28 @@ __global__ void __launch_bounds__(32 * wide_max_warps<E>(), 1)
         word |= ((y | (y >> 15)) & 0xffu) << (8 * u);
       }
       mw[(k << 5) | lane] = word;
-      // high bit of every non-zero byte, then those four bits gathered into
-      // bits 28..31 by one multiply (the partial products do not overlap)
-      const uint32_t nz = (((word & 0x7f7f7f7fu) + 0x7f7f7f7fu) | word) & 0x80808080u;
-      hits |= ((nz * 0x00204081u) >> 28) << (4 * k);
+      hits |= (word != 0u ? 1u : 0u) << k;
     }
 
     // ---- C: exact top-(K+1) of the experts with a hit, in ascending index,
-    // one per lane per step; the next candidate's z and b are read one step
-    // ahead.  Refills are branch-free, and a lane that is done inserts -inf,
-    // which leaves its list unchanged.
+    // one per lane per step, taken from the mask words 32 experts at a time;
+    // the next candidate's z and b are read one step ahead.  Refills are
+    // branch-free, and a lane that is done inserts -inf, which leaves its
+    // list unchanged.
     float v[KP1];
     int id[KP1];
 #pragma unroll
     for (int j = 0; j < KP1; ++j) { v[j] = -INFINITY; id[j] = 0; }
-    int cb = 0;
+    int wb = 0;  // first expert of the current mask word
     uint32_t m = 0u;
     auto fetch = [&]() -> int {
       const bool need = m == 0u && hits != 0u;
-      const int c = __ffs(hits) - 1;
-      const int cc = need ? c : 0;
-      const uint32_t word = mw[((cc >> 2) << 5) | lane];
-      m = need ? (word >> ((cc & 3) << 3)) & 0xffu : m;
-      cb = need ? c << 3 : cb;
+      const int k = __ffs(hits) - 1;
+      const uint32_t word = mw[((need ? k : 0) << 5) | lane];
+      m = need ? word : m;
+      wb = need ? k << 5 : wb;
       hits = need ? hits & (hits - 1u) : hits;
-      const int e = m != 0u ? cb + __ffs(m) - 1 : -1;
+      const int e = m != 0u ? wb + __ffs(m) - 1 : -1;
       m &= m - 1u;
       return e;
     };
