@@ -136,3 +136,38 @@ def test_layer_step_at_and_past_the_coefficient_table(T, E, K, M):
     assert np.array_equal(loads.cpu().numpy(), o["loads"])
     assert np.array_equal(bits_f32(bn.cpu().numpy()), bits_f32(o["b_next"]))
     assert within(G.view.cpu().numpy(), g_ref)
+
+
+@pytest.mark.parametrize("T", [1, 2, 3, 31, 33, 1025])
+@pytest.mark.parametrize("E,K", [(8, 2), (64, 8), (256, 8)])
+def test_layer_step_tiny_batches_with_lei(T, E, K):
+    """Batches smaller than a warp round, a histogram block or a LEI chunk
+    (an empty first half at T = 1) through the fused step."""
+    rng = np.random.default_rng(T * 1000 + E)
+    z = brute.bf16_bits_from_f32(rng.standard_normal((T, E)).astype(np.float32))
+    b = (rng.standard_normal(E) * 0.3).astype(np.float32)
+    off = np.array([0, T // 2, T], np.int64) if T >= 2 else np.array([0, T], np.int64)
+    M = len(off) - 1
+    g = (rng.standard_normal((T, E)) * 0.1).astype(np.float32)
+    eta, c = 0.5, 2.0
+    o = oracle_forward(z, b, K, off)
+    g_ref, _ = oracle.lei(g, o["loads"], off, K, eta, c)
+    idx = Guarded((T, K), torch.int32)
+    tau = Guarded((T,), torch.float32)
+    loads = Guarded((M, E), torch.int32, fill=5)
+    bn = Guarded((E,), torch.float32)
+    G = Guarded((T, E), torch.float32)
+    G.view.copy_(torch.from_numpy(g))
+    ws = torch.zeros(eqb.eqb_layer_workspace_bytes(E), dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    eqb.eqb_layer_step(to_dev_bf16(z), torch.from_numpy(b).cuda(), K, torch.from_numpy(off).cuda(), loads.view,
+                       bn.view, ws, tau=tau.view, topk_idx=idx.view, grad_s=G.view, eta=eta, c=c,
+                       mb_offsets_host=off, err_flag=err)
+    torch.cuda.synchronize()
+    for buf in (idx, tau, loads, bn, G):
+        assert buf.intact()
+    assert err.item() == 0
+    assert np.array_equal(idx.view.cpu().numpy(), o["idx"])
+    assert np.array_equal(loads.view.cpu().numpy(), o["loads"])
+    assert np.array_equal(bits_f32(bn.view.cpu().numpy()), bits_f32(o["b_next"]))
+    assert within(G.view.cpu().numpy(), g_ref)
