@@ -105,6 +105,40 @@ def test_lei_rejects(lib):
     assert f(FAKE, FAKE, FAKE, 1, 0, 64, 8, ctypes.c_float(1.0), ctypes.c_float(1.0), NULL) == 0
 
 
+def test_lei_coefficients_rejects(lib):
+    f = lib.lei_coefficients
+    one = ctypes.c_float(1.0)
+    assert f(NULL, FAKE, 1, 64, 8, one, one, FAKE, NULL) == INVALID
+    assert f(FAKE, FAKE, 0, 64, 8, one, one, FAKE, NULL) == INVALID
+    assert f(FAKE, FAKE, 1, 64, 8, one, one, NULL, NULL) == INVALID
+    assert f(FAKE, FAKE, 1, 64, 8, one, one, MISALIGNED, NULL) == INVALID
+    assert f(FAKE, FAKE, 1, 64, 64, one, one, FAKE, NULL) == INVALID  # K >= E
+    assert f(FAKE, FAKE, 1, 64, 8, ctypes.c_float(float("nan")), one, FAKE, NULL) == INVALID
+    assert f(FAKE, FAKE, 1, 2048, 8, one, one, FAKE, NULL) == UNSUPPORTED
+
+
+def test_fused_pass_rejects(lib):
+    f = lib.eqb_margin_hist_lei
+
+    def call(T=100, E=64, pass_=1, u=FAKE, grad=FAKE, coef=FAKE, off=FAKE, M=1, t0=0, t1=100, z=FAKE):
+        return f(z, FAKE, T, E, pass_, u, FAKE, NULL, grad, coef, off, M, t0, t1, NULL)
+
+    assert call(pass_=3) == INVALID
+    assert call(pass_=2, u=NULL) == INVALID
+    assert call(grad=NULL) == INVALID
+    assert call(coef=NULL) == INVALID
+    assert call(off=NULL) == INVALID
+    assert call(M=0) == INVALID
+    assert call(t0=-1) == INVALID
+    assert call(t0=50, t1=40) == INVALID
+    assert call(t1=101) == INVALID
+    assert call(grad=MISALIGNED) == INVALID
+    assert call(coef=MISALIGNED) == INVALID
+    assert call(z=MISALIGNED) == INVALID
+    assert call(E=12) == UNSUPPORTED
+    assert call(T=0, t1=0) == 0
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     from paper_2609_28053_gb300 import _lib
     with pytest.raises(RuntimeError, match="no CPU fallback"):
