@@ -186,6 +186,50 @@ def test_global_config_full_size_sampled():
 
 
 @pytest.mark.slow
+@pytest.mark.parametrize("name", ["global", "paper"])
+def test_layer_step_full_size(name):
+    """The benchmark's timed call at full size (eqb_layer_step on the global
+    workload, T = 2,097,152, E = 256, K = 8, M = 64, and on the paper's shape,
+    T = 9,437,184, K = 6; LEI streamed inside the histogram passes, eta and c
+    of the benchmark): every token's top-K and cutoff, all loads and the next
+    bias of all 256 experts bit for bit against the oracle (full-sort
+    quantiles), and 4,096 sampled rows of the injected gradient within the
+    LEI tolerance of the oracle's coefficients."""
+    sh = SHAPES[name]
+    T, E, K, M = sh.T, sh.E, sh.K, sh.M
+    eta, c = 2e-5, 1.0
+    zt = make_logits(name, device="cuda")
+    bt = make_bias(name, device="cuda")
+    G = make_grad(name, device="cuda")
+    rows = np.sort(np.random.default_rng(5).choice(T, 4096, replace=False))
+    rows_d = torch.from_numpy(rows).cuda()
+    g_rows = G[rows_d].cpu().numpy()
+    off = even_offsets(T, M)
+    offd = torch.from_numpy(off).cuda()
+    idx = torch.empty((T, K), dtype=torch.int32, device="cuda")
+    tau = torch.empty(T, dtype=torch.float32, device="cuda")
+    loads = torch.zeros((M, E), dtype=torch.int32, device="cuda")
+    bn = torch.empty(E, dtype=torch.float32, device="cuda")
+    ws = torch.zeros(eqb.eqb_layer_workspace_bytes(E), dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    eqb.eqb_layer_step(zt, bt, K, offd, loads, bn, ws, tau=tau, topk_idx=idx, grad_s=G, eta=eta, c=c,
+                       mb_offsets_host=off, err_flag=err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    got_rows = G[rows_d].cpu().numpy()
+    z = bits(zt)
+    o = oracle_forward(z, bt.cpu().numpy(), K, off, experts=np.arange(E))
+    assert np.array_equal(idx.cpu().numpy(), o["idx"])
+    assert np.array_equal(bits_f32(tau.cpu().numpy()), bits_f32(o["tau"]))
+    assert np.array_equal(loads.cpu().numpy(), o["loads"])
+    assert np.array_equal(bits_f32(bn.cpu().numpy()), bits_f32(oracle.bias_update(o["q"])))
+    _, a = oracle.lei(None, o["loads"], off, K, eta, c)
+    mb = np.searchsorted(off, rows, side="right") - 1
+    want = g_rows.astype(np.float64) + a[mb]
+    assert np.all(np.abs(got_rows.astype(np.float64) - want) <= LEI_ATOL + LEI_RTOL * np.abs(want))
+
+
+@pytest.mark.slow
 def test_paper_config_full_size_sampled():
     """The paper's own shape (Sec. 5 / App. E.1: E = 256, K = 6, 147,456 tokens
     on each of 64 ranks, T = 9,437,184): every token's top-K and cutoff, all
