@@ -502,7 +502,7 @@ def main():
     ap.add_argument("--steps", type=int, default=100)
     ap.add_argument("--warmup", type=int, default=5)
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
-    ap.add_argument("--workload", default="global", choices=["global", "router", "paper"])
+    ap.add_argument("--workload", default="global", choices=["global", "router", "paper", "wide"])
     ap.add_argument("--tokens", type=int, default=None)
     ap.add_argument("--e2e-steps", type=int, default=8)
     ap.add_argument("--cpu-sample-tokens", type=int, default=131072)

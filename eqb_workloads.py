@@ -23,6 +23,8 @@ Shapes (token count T, experts E, experts per token K, microbatches M):
   paper   T=9,437,184  E=256  K=6  M=64 x 147,456 z ~ N(0,1); b ~ N(0, 0.2^2)
           (the paper's own setting, Sec. 5 / App. E.1: 256 experts, top-6,
           147,456 tokens per data-parallel rank, 64 ranks)
+  wide    T=1,048,576  E=512  K=8  M=32 x 32,768  z ~ N(0,1); b ~ N(0, 0.2^2)
+          (more experts than one histogram block holds)
 
 Upstream router-score gradients g ~ N(0, 0.1^2) fp32 (variance 1e-2) for
 every config.  Logits are rounded to bf16 round-to-nearest-even by torch.
@@ -39,7 +41,7 @@ from dataclasses import dataclass, field
 import numpy as np
 import torch
 
-CONFIG_NAMES = ("tiny", "tie", "mid", "global", "router", "paper")
+CONFIG_NAMES = ("tiny", "tie", "mid", "global", "router", "paper", "wide")
 
 
 @dataclass(frozen=True)
@@ -62,6 +64,8 @@ SHAPES = {
     "global": Shape("global", 2097152, 256, 8, 64, seed=1003),
     "router": Shape("router", 1048576, 128, 8, 16, d=4096, steps=3, seed=1004),
     "paper": Shape("paper", 9437184, 256, 6, 64, seed=1005),
+    # more experts than one histogram block holds (expert-tiled passes)
+    "wide": Shape("wide", 1048576, 512, 8, 32, seed=1006),
 }
 
 
@@ -123,7 +127,7 @@ def make_logits(name: str, T: int | None = None, seed: int | None = None,
     seed = sh.seed if seed is None else seed
     E = sh.E
     d = _Draw(seed, device)
-    if name in ("tiny", "router", "paper"):
+    if name in ("tiny", "router", "paper", "wide"):
         return _bf16(d.normal((T, E)))
     if name == "tie":
         mu = d.normal((E,)) * 0.5
@@ -153,7 +157,7 @@ def make_bias(name: str, seed: int | None = None, device: str = "cpu") -> torch.
     d = _Draw(seed, device)
     if name == "tie":
         return d.uniform((sh.E,), -0.1, 0.1)
-    if name in ("global", "paper"):
+    if name in ("global", "paper", "wide"):
         return d.normal((sh.E,)) * 0.2
     return torch.zeros(sh.E, dtype=torch.float32, device=device)
 

@@ -1,6 +1,7 @@
 // route_wide.cu -- top-K routing, cutoff tau_t and per-microbatch loads
 // (Sec. 2, Eq. 1 and the QB paragraph of arXiv 2609.28053) for the wide rows
-// E = 128 and E = 256 with K + 1 <= 16, the row width fixed at compile time.
+// E = 128, 256, 384 and 512 with K + 1 <= 16, the row width fixed at compile
+// time.
 //
 // One thread owns one token; a warp owns a tile of 32 consecutive tokens,
 // which each lane brings into shared memory with one bulk copy of its row
@@ -80,6 +81,7 @@ __global__ void __launch_bounds__(32 * wide_max_warps<E>(), 1)
     route_wide_kernel(RouteArgs a, int64_t tiles_per_warp) {
   using L = WideLayout<E>;
   constexpr int NCH = L::NCH, NH = NCH / 2;
+  constexpr int NP = NH <= 8 ? 8 : NH <= 16 ? 16 : 32;  // sorted length (a power of two)
   extern __shared__ __align__(16) uint8_t smem[];
   const int K = a.K;
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5;
@@ -172,10 +174,16 @@ __global__ void __launch_bounds__(32 * wide_max_warps<E>(), 1)
     const int64_t t = (tl << 5) + lane;
     const bool valid = t < a.T;
 
-    // ---- A: chunk maxima of L, chunks c and c + NH in one word
-    uint32_t cm[NH];
+    // ---- A: chunk maxima of L, chunks c and c + NH in one word (words past
+    // NH, when NH is not a power of two, hold -inf in both halves)
+    uint32_t cm[NP];
+#pragma unroll
+    for (int c = NH; c < NP; ++c) cm[c] = 0xff80ff80u;
 #pragma unroll
     for (int c = 0; c < NH; ++c) {
+      // At E > 256 the unrolled loads would not fit in registers if all were
+      // hoisted: let at most eight pairs of chunks be in flight.
+      if (NH > 16 && c > 0 && (c & 7) == 0) asm volatile("" ::: "memory");
       const uint32_t qa = chunk_max(lds128(rowp + 16 * c), bdn4[c]);
       const uint32_t qb = chunk_max(lds128(rowp + 16 * (c + NH)), bdn4[c + NH]);
       cm[c] = hmax2_nan_bf16(prmt(qa, qb, 0x5410u), prmt(qa, qb, 0x7632u));
@@ -185,13 +193,13 @@ __global__ void __launch_bounds__(32 * wide_max_warps<E>(), 1)
     for (int c = 1; c < NH; ++c) anynan = hmax2_nan_bf16(anynan, cm[c]);
     if (valid && ((anynan & 0x7fffu) > 0x7f80u || (anynan >> 16 & 0x7fffu) > 0x7f80u))
       raise_flag(a.err, kErrNonfinite);
-    sort_desc_bf16x2<NH>(cm);
+    sort_desc_bf16x2<NP>(cm);
     float theta = INFINITY;
 #pragma unroll
     for (int i = 0; i < KP1; ++i) {
       const int j = KP1 - 1 - i;
-      const float x = i < NH ? bf16_lo(cm[i < NH ? i : 0]) : -INFINITY;
-      const float y = j < NH ? bf16_hi(cm[j < NH ? j : 0]) : -INFINITY;
+      const float x = i < NP ? bf16_lo(cm[i < NP ? i : 0]) : -INFINITY;
+      const float y = j < NP ? bf16_hi(cm[j < NP ? j : 0]) : -INFINITY;
       theta = fminf(theta, fmaxf(x, y));
     }
     // Near zero, flushing of subnormal bf16 sums could move L by up to
@@ -350,11 +358,15 @@ int launch_wide_e(const RouteArgs& a, cudaStream_t s) {
 
 }  // namespace
 
-bool route_wide_supported(int E, int K) { return (E == 128 || E == 256) && K + 1 <= 16; }
+bool route_wide_supported(int E, int K) {
+  return (E == 128 || E == 256 || E == 384 || E == 512) && K + 1 <= 16;
+}
 
 int launch_route_wide(const RouteArgs& a, cudaStream_t s) {
   if (a.E == 256) return launch_wide_e<256>(a, s);
   if (a.E == 128) return launch_wide_e<128>(a, s);
+  if (a.E == 512) return launch_wide_e<512>(a, s);
+  if (a.E == 384) return launch_wide_e<384>(a, s);
   return kErrUnsupported;
 }
 

@@ -186,15 +186,16 @@ def test_global_config_full_size_sampled():
 
 
 @pytest.mark.slow
-@pytest.mark.parametrize("name", ["global", "paper"])
+@pytest.mark.parametrize("name", ["global", "paper", "wide"])
 def test_layer_step_full_size(name):
     """The benchmark's timed call at full size (eqb_layer_step on the global
-    workload, T = 2,097,152, E = 256, K = 8, M = 64, and on the paper's shape,
-    T = 9,437,184, K = 6; LEI streamed inside the histogram passes, eta and c
-    of the benchmark): every token's top-K and cutoff, all loads and the next
-    bias of all 256 experts bit for bit against the oracle (full-sort
-    quantiles), and 4,096 sampled rows of the injected gradient within the
-    LEI tolerance of the oracle's coefficients."""
+    workload, T = 2,097,152, E = 256, K = 8, M = 64, on the paper's shape,
+    T = 9,437,184, K = 6, and on the wide workload, T = 1,048,576, E = 512;
+    LEI streamed inside the histogram passes, eta and c of the benchmark):
+    every token's top-K and cutoff, all loads and the next bias of every
+    expert bit for bit against the oracle (full-sort quantiles), and 4,096
+    sampled rows of the injected gradient within the LEI tolerance of the
+    oracle's coefficients."""
     sh = SHAPES[name]
     T, E, K, M = sh.T, sh.E, sh.K, sh.M
     eta, c = 2e-5, 1.0
