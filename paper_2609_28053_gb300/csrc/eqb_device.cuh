@@ -297,4 +297,94 @@ __device__ __forceinline__ bool bar_wait_bounded(uint32_t bar, uint32_t parity, 
     if (bar_try_wait(bar, parity)) return true;
   return false;
 }
+
+// ---- Load-Error Injection streamed by one warp (Sec. 4, Eq. LEI), used by
+// the histogram passes that carry LEI beside their counting.
+
+// Token slice [q0, q1) of block `cta` out of `nct` blocks over [t0, t1).
+__device__ __forceinline__ void lei_block_slice(int64_t t0, int64_t t1, int64_t cta, int64_t nct, int64_t* q0,
+                                                int64_t* q1) {
+  const int64_t n = t1 - t0;
+  const int64_t per = (n + nct - 1) / nct;
+  *q0 = t0 + min(cta * per, n);
+  *q1 = t0 + min(cta * per + per, n);
+}
+
+// One warp adds coef[mb(t), e] to grad_s[t, e] for the tokens [ta, tb), in
+// fp32 round to nearest, with evict-first 16-byte loads and stores and
+// U loads in flight per lane.  (mlo, mhi, ml) caches the token range of
+// the last microbatch looked up (start with mlo > mhi).  Tokens past the
+// last boundary (malformed offsets) are the last microbatch's.
+template <int U = 8>
+__device__ __forceinline__ void lei_warp_tokens(const LeiStream& ls, int E, int64_t ta, int64_t tb, int64_t& mlo,
+                                                int64_t& mhi, int& ml) {
+  const int lane = threadIdx.x & 31;
+  const int E4 = E >> 2;
+  const int dcol = 32 % E4;
+  float4* g4 = reinterpret_cast<float4*>(ls.g);
+  const float4* c4 = reinterpret_cast<const float4*>(ls.coef);
+  while (ta < tb) {
+    if (ta < mlo || ta >= mhi) {
+      ml = microbatch_of(ls.off, ls.M, ta);
+      mlo = __ldg(ls.off + ml);
+      mhi = __ldg(ls.off + ml + 1);
+    }
+    const int64_t se = mhi > ta ? min(tb, mhi) : tb;
+    const float4* crow = c4 + (int64_t)ml * E4;
+    int64_t i = ta * E4 + lane;
+    const int64_t i1 = se * E4;
+    int col = static_cast<int>(i % E4);
+    for (; i + 32 * (U - 1) < i1; i += 32 * U) {
+      float4 v[U];
+      int cc[U];
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        v[u] = __ldcs(g4 + i + 32 * u);
+        cc[u] = col;
+        col += dcol;
+        if (col >= E4) col -= E4;
+      }
+#pragma unroll
+      for (int u = 0; u < U; ++u) {
+        const float4 cf = __ldg(crow + cc[u]);
+        v[u].x = __fadd_rn(v[u].x, cf.x);
+        v[u].y = __fadd_rn(v[u].y, cf.y);
+        v[u].z = __fadd_rn(v[u].z, cf.z);
+        v[u].w = __fadd_rn(v[u].w, cf.w);
+        __stcs(g4 + i + 32 * u, v[u]);
+      }
+    }
+    for (; i < i1; i += 32) {
+      float4 v = __ldcs(g4 + i);
+      const float4 cf = __ldg(crow + col);
+      v.x = __fadd_rn(v.x, cf.x);
+      v.y = __fadd_rn(v.y, cf.y);
+      v.z = __fadd_rn(v.z, cf.z);
+      v.w = __fadd_rn(v.w, cf.w);
+      __stcs(g4 + i, v);
+      col += dcol;
+      if (col >= E4) col -= E4;
+    }
+    ta = se;
+  }
+}
+
+// Tokens per chunk of a block's LEI slice: about 8 KiB of grad_s.
+__device__ __forceinline__ int lei_chunk_tokens(int E) { return max(1, 2048 / E); }
+
+// One warp takes the next chunk of [q0, q1) through the block's shared
+// counter *next and streams it (U loads in flight per lane); false when the
+// slice is used up.
+template <int U = 8>
+__device__ __forceinline__ bool lei_warp_next_chunk(const LeiStream& ls, int E, int64_t q0, int64_t q1, int* next,
+                                                    int64_t& mlo, int64_t& mhi, int& ml) {
+  int c = 0;
+  if ((threadIdx.x & 31) == 0) c = atomicAdd(next, 1);
+  c = __shfl_sync(kFull, c, 0);
+  const int ch = lei_chunk_tokens(E);
+  const int64_t ta = q0 + (int64_t)c * ch;
+  if (ta >= q1) return false;
+  lei_warp_tokens<U>(ls, E, ta, min(ta + ch, q1), mlo, mhi, ml);
+  return true;
+}
 }  // namespace eqb

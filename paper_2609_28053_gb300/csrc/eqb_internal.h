@@ -25,6 +25,17 @@ struct DeviceInfo {
 // Cached per-device attributes (queried once per device).
 int device_info(DeviceInfo* out);
 
+// Load-Error Injection streamed by a histogram pass beside its own work:
+// grad_s[t, e] += coef[mb(t), e] for the tokens [t0, t1), from the [M,E]
+// coefficient table of launch_lei_coef.  Token numbers are absolute.
+struct LeiStream {
+  float* g = nullptr;  // nullptr: no injection
+  const float* coef = nullptr;
+  const int64_t* off = nullptr;
+  int M = 0;
+  int64_t t0 = 0, t1 = 0;
+};
+
 struct RouteArgs {
   const uint16_t* z;
   const float* b;
@@ -67,17 +78,6 @@ struct LeiArgs {
   int64_t T;
   int E, K;
   float eta, c;
-};
-
-// Load-Error Injection streamed by a histogram pass beside its own work:
-// grad_s[t, e] += coef[mb(t), e] for the tokens [t0, t1), from the [M,E]
-// coefficient table of launch_lei_coef.  Token numbers are absolute.
-struct LeiStream {
-  float* g = nullptr;  // nullptr: no injection
-  const float* coef = nullptr;
-  const int64_t* off = nullptr;
-  int M = 0;
-  int64_t t0 = 0, t1 = 0;
 };
 
 struct GshardArgs {

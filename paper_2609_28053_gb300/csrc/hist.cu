@@ -44,80 +44,17 @@ namespace {
 
 constexpr int kUnroll = 8;  // 16-byte loads in flight per lane (64 registers at 1024 threads)
 constexpr int64_t kFlushTokens = 65535;
-constexpr int kLeiUnroll = 8;  // 16-byte grad_s loads in flight per lane in the injection stream
-
 // The injection share of a fused block (see above): chunks of about 8 KiB of
 // grad_s from this block's slice of [ls.t0, ls.t1), taken through the shared
 // counter *next.  Every element gets one fp32 addition (round to nearest) of
 // its microbatch's coefficient, as in lei.cu.
 __device__ __forceinline__ void stream_lei(const LeiStream& ls, int E, int* next) {
-  const int lane = threadIdx.x & 31;
-  const int64_t nct = (int64_t)gridDim.x * gridDim.y;
-  const int64_t cta = (int64_t)blockIdx.y * gridDim.x + blockIdx.x;
-  const int64_t n = ls.t1 - ls.t0;
-  const int64_t per = (n + nct - 1) / nct;
-  const int64_t q0 = ls.t0 + min(cta * per, n);
-  const int64_t q1 = ls.t0 + min(cta * per + per, n);
-  const int E4 = E >> 2;
-  const int ch = max(1, 512 / E4);  // tokens per chunk
-  const int dcol = 32 % E4;
-  float4* g4 = reinterpret_cast<float4*>(ls.g);
-  const float4* c4 = reinterpret_cast<const float4*>(ls.coef);
+  int64_t q0, q1;
+  lei_block_slice(ls.t0, ls.t1, (int64_t)blockIdx.y * gridDim.x + blockIdx.x, (int64_t)gridDim.x * gridDim.y, &q0,
+                  &q1);
   int64_t mlo = 1, mhi = 0;  // token range of microbatch ml (none yet)
   int ml = 0;
-  for (;;) {
-    int c = 0;
-    if (lane == 0) c = atomicAdd(next, 1);
-    c = __shfl_sync(kFull, c, 0);
-    int64_t ta = q0 + (int64_t)c * ch;
-    if (ta >= q1) break;
-    const int64_t tb = min(ta + ch, q1);
-    while (ta < tb) {
-      if (ta < mlo || ta >= mhi) {
-        ml = microbatch_of(ls.off, ls.M, ta);
-        mlo = __ldg(ls.off + ml);
-        mhi = __ldg(ls.off + ml + 1);
-      }
-      // Malformed offsets (off[M] < T): tokens past the last boundary are
-      // the last microbatch's, as in lei.cu.
-      const int64_t se = mhi > ta ? min(tb, mhi) : tb;
-      const float4* crow = c4 + (int64_t)ml * E4;
-      int64_t i = ta * E4 + lane;
-      const int64_t i1 = se * E4;
-      int col = static_cast<int>(i % E4);
-      for (; i + 32 * (kLeiUnroll - 1) < i1; i += 32 * kLeiUnroll) {
-        float4 v[kLeiUnroll];
-        int cc[kLeiUnroll];
-#pragma unroll
-        for (int u = 0; u < kLeiUnroll; ++u) {
-          v[u] = __ldcs(g4 + i + 32 * u);
-          cc[u] = col;
-          col += dcol;
-          if (col >= E4) col -= E4;
-        }
-#pragma unroll
-        for (int u = 0; u < kLeiUnroll; ++u) {
-          const float4 cf = __ldg(crow + cc[u]);
-          v[u].x = __fadd_rn(v[u].x, cf.x);
-          v[u].y = __fadd_rn(v[u].y, cf.y);
-          v[u].z = __fadd_rn(v[u].z, cf.z);
-          v[u].w = __fadd_rn(v[u].w, cf.w);
-          __stcs(g4 + i + 32 * u, v[u]);
-        }
-      }
-      for (; i < i1; i += 32) {
-        float4 v = __ldcs(g4 + i);
-        const float4 cf = __ldg(crow + col);
-        v.x = __fadd_rn(v.x, cf.x);
-        v.y = __fadd_rn(v.y, cf.y);
-        v.z = __fadd_rn(v.z, cf.z);
-        v.w = __fadd_rn(v.w, cf.w);
-        __stcs(g4 + i, v);
-        col += dcol;
-        if (col >= E4) col -= E4;
-      }
-      ta = se;
-    }
+  while (lei_warp_next_chunk(ls, E, q0, q1, next, mlo, mhi, ml)) {
   }
 }
 
