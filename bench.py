@@ -512,7 +512,8 @@ def main():
     ap.add_argument("--workload", default="global", choices=["global", "router", "paper", "wide"])
     ap.add_argument("--tokens", type=int, default=None)
     ap.add_argument("--e2e-steps", type=int, default=8)
-    ap.add_argument("--cpu-sample-tokens", type=int, default=131072)
+    # the oracle's CPU baseline sample: about 10 s of one host core
+    ap.add_argument("--cpu-sample-tokens", type=int, default=294912)
     ap.add_argument("--ref-sample-tokens", type=int, default=32768)
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-extras", action="store_true")
@@ -668,7 +669,7 @@ def main():
 
     cpu_base = None
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        n = min(args.cpu_sample_tokens if args.workload != "router" else 8192, T)
+        n = min(args.cpu_sample_tokens if args.workload != "router" else 18432, T)
         if args.workload == "router":
             secs, toks = cpu_oracle_router_sample(step.x, step.W, step.g, K, n)
             what = (f"first {n} tokens: router projection in fp64, routing, exact quantile of all "
