@@ -2,8 +2,12 @@
 // order of launches; every step runs in the library's kernels).
 //
 // Order of work, as in the paper: routing (Sec. 2), Algorithm 1's coarse
-// pass, selection, fine pass, selection and the Eq. (2) bias update, then
-// Load-Error Injection (Sec. 4, Eqs. LEI and norm).  All on one stream.
+// pass, selection, fine pass, selection and the Eq. (2) bias update, and
+// Load-Error Injection (Sec. 4, Eqs. LEI and norm).  LEI needs only the
+// loads, so when its [M,E] coefficient table fits the workspace the
+// coefficients are formed right after routing and the two histogram passes
+// stream the injection, half of the tokens each; otherwise it runs last.
+// All on one stream.
 // eqb_router_layer_step starts one step earlier, at the router projection
 // (Eq. 1), and routes from the projection's accumulators where it can.
 #include <cuda_runtime.h>
