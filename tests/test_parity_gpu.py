@@ -61,8 +61,10 @@ def test_forward_small_shapes(T, E, K):
 @pytest.mark.parametrize("T", [33, 1000])
 @pytest.mark.parametrize("E,K", [(264, 8), (384, 8), (512, 6), (1024, 8), (1024, 31)])
 def test_forward_many_experts(T, E, K):
-    """E above 256: the generic routing kernel, histograms tiled over
-    experts, selection and the bias update on up to 1024 experts."""
+    """E above 256: the compile-time-width routing kernel (E = 384, 512 with
+    K + 1 <= 16) and the runtime-width one (E = 264, 1024, and K = 31),
+    histograms tiled over experts, selection and the bias update on up to
+    1024 experts."""
     z, b = rand_case(T, E, seed=T + E + K)
     off = ragged_offsets(T, 3, seed=E)
     assert_forward_equal(gpu_forward(z, b, K, off), oracle_forward(z, b, K, off))
