@@ -461,6 +461,32 @@ def extras(step, stream, peak):
     row("fixed_hist_bias", time_call(lambda: eqb.eqb_fixed_hist_bias(
         z, step.tau, K, lo, width, step.workspace, stream=stream), stream), 2 * T * E + 4 * T)
 
+    # Routing with the coarse histogram: the one-read kernel against the two
+    # kernels the step uses (routing, then the coarse pass), same outputs.
+    if E in (128, 256) and K + 1 <= 16:
+        ws = step.ws
+        idx2 = torch.empty_like(step.idx)
+        tau2 = torch.empty_like(step.tau)
+        ld2 = torch.zeros_like(step.loads)
+
+        def two_kernels():
+            ws.hist_hi.zero_()
+            ld2.zero_()
+            eqb.eqb_route_topk(z, step.b, K, off, idx2, tau2, ld2, ws.hist_hi, None, stream)
+
+        def one_kernel():
+            ws.hist_hi.zero_()
+            ld2.zero_()
+            eqb.eqb_route_hist_fused(z, step.b, K, off, idx2, tau2, ld2, ws.hist_hi, None, stream)
+
+        zero_ms = time_call(lambda: (ws.hist_hi.zero_(), ld2.zero_()), stream)
+        two = time_call(two_kernels, stream) - zero_ms
+        one = time_call(one_kernel, stream) - zero_ms
+        out["route_and_coarse_hist"] = {
+            "two_kernels_ms": round(two, 5), "one_read_kernel_ms": round(one, 5),
+            "two_kernels_bytes": 2 * (2 * T * E) + 4 * T * K + 8 * T,
+            "one_read_bytes": 2 * T * E + 4 * T * K + 4 * T}
+
     # Balance after one update: each bias routes a fresh batch.
     b0 = step.b.clone()
     loads = torch.zeros_like(step.loads)

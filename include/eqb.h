@@ -95,11 +95,27 @@ int64_t eqb_target_rank(int64_t T, int32_t E, int32_t K);
  *   hist_hi   device int32 [E,256] += (nullable)           (in/out)
  *   err_flag  device int32 (nullable): EQB_ERR_NONFINITE for a non-finite
  *             b_e or NaN score, or (with hist_hi) a non-finite margin.
+ *
+ * With hist_hi the coarse pass runs as a second kernel over z (on GB300 the
+ * two kernels are faster than the one-read eqb_route_hist_fused).
  */
 eqb_status eqb_route_topk(const eqb_bf16 *z, const float *b, int64_t T, int32_t E,
                           int32_t K, const int64_t *mb_offsets, int32_t M,
                           int32_t *topk_idx, float *tau, int32_t *loads,
                           int32_t *hist_hi, int32_t *err_flag, void *stream);
+
+/* Routing and the coarse pass in one pass over z (Sec. 2 Eq. 1 and the QB
+ * paragraph; Algorithm 1 step 1): the results of eqb_route_topk with hist_hi,
+ * from one kernel that routes each 32-token tile staged in shared memory and
+ * then counts the same staged tile, so z is read from DRAM once instead of
+ * twice.  E = 128 or 256 and K + 1 <= 16, else EQB_ERR_UNSUPPORTED.
+ * Arguments as in eqb_route_topk; hist_hi is required.  Bit-identical
+ * outputs; slower than the two kernels on GB300, where both are bound by
+ * instruction issue rather than by DRAM. */
+eqb_status eqb_route_hist_fused(const eqb_bf16 *z, const float *b, int64_t T, int32_t E,
+                                int32_t K, const int64_t *mb_offsets, int32_t M,
+                                int32_t *topk_idx, float *tau, int32_t *loads,
+                                int32_t *hist_hi, int32_t *err_flag, void *stream);
 
 /* Coarse pass on its own (Algorithm 1 step 1): recomputes the margins from z
  * and tau and accumulates hist_hi[e, kappa(m) >> 8] += 1 over T tokens.
@@ -186,7 +202,7 @@ eqb_status eqb_margin_hist_lei(const eqb_bf16 *z, const float *tau, int64_t T,
 
 /* Bytes of device workspace eqb_layer_step needs for E experts (the two
  * [E,256] histograms, u, rho, q_hat and a 65,536-float LEI coefficient
- * table, each 256-byte aligned). */
+ * table, each 256-byte aligned; 788,224 bytes for E = 256). */
 size_t eqb_layer_workspace_bytes(int32_t E);
 
 /* One layer's whole routing-balance step in one call, in the paper's order:
@@ -221,12 +237,16 @@ eqb_status eqb_layer_step(const eqb_bf16 *z, const float *b, int64_t T, int32_t 
  * code that must not stall on or fail at an allocation, can call this
  * instead: it takes the same inputs and outputs but no workspace, and uses a
  * scratch array compiled into the library.
- *   - The scratch holds the step's histograms and selections for E <= 256
- *     (526,080 bytes); E > 256 returns EQB_ERR_UNSUPPORTED.  Every GPU that
- *     loads the library keeps this array until the process exits.
+ *   - The scratch is eqb_layer_workspace_bytes(256) = 788,224 bytes: the
+ *     step's two histograms, u, rho, q_hat and the 65,536-float LEI
+ *     coefficient table, enough for E <= 256; E > 256 returns
+ *     EQB_ERR_UNSUPPORTED.  Every GPU that loads the library keeps
+ *     this array until the process exits.
  *   - The first call on each device looks up the array's device address
  *     (cudaGetSymbolAddress) with that device current; make it before any
- *     stream capture.  It allocates nothing.
+ *     stream capture.  It allocates nothing.  The address is kept for the
+ *     life of the process: after cudaDeviceReset on that device it is stale,
+ *     and calls must not be made there again.
  *   - All calls on a device share the array, which keeps the previous
  *     call's contents (the step zeroes the histograms before counting);
  *     calls that overlap on the GPU race on it.

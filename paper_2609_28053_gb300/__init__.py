@@ -63,6 +63,15 @@ def _need(t, dtype, name, shape=None):
         raise ValueError(f"{name} must have shape {tuple(shape)}, got {tuple(t.shape)}")
 
 
+def _on_current_device(t, name):
+    """The library takes its scratch and streams from the CUDA device that is
+    current when it is called: the tensors must live on that device."""
+    cur = torch.cuda.current_device()
+    if t.device.index != cur:
+        raise ValueError(f"{name} is on cuda:{t.device.index} but cuda:{cur} is the current device; "
+                         f"call inside torch.cuda.device({t.device})")
+
+
 def _check(rc, what):
     if rc != 0:
         raise EqbError(rc, what)
@@ -95,6 +104,31 @@ def eqb_route_topk(z, b, K, mb_offsets=None, topk_idx=None, tau=None, loads=None
                                _p(loads), _p(hist_hi), _p(err_flag), _stream(stream))
     _check(rc, "eqb_route_topk")
     return topk_idx, tau
+
+
+def eqb_route_hist_fused(z, b, K, mb_offsets=None, topk_idx=None, tau=None, loads=None, hist_hi=None,
+                         err_flag=None, stream=None):
+    """Routing and the coarse histogram from one kernel that reads z once
+    (E = 128 or 256): the outputs of eqb_route_topk with hist_hi, bit for
+    bit.  Returns tau."""
+    T, E = z.shape
+    _need(z, torch.bfloat16, "z")
+    _need(b, torch.float32, "b", (E,))
+    if tau is None:
+        tau = torch.empty(T, dtype=torch.float32, device=z.device)
+    _need(tau, torch.float32, "tau", (T,))
+    _need(topk_idx, torch.int32, "topk_idx", (T, K))
+    _need(mb_offsets, torch.int64, "mb_offsets")
+    M = 0 if mb_offsets is None else mb_offsets.numel() - 1
+    _need(loads, torch.int32, "loads", (M, E) if loads is not None else None)
+    _need(hist_hi, torch.int32, "hist_hi", (E, 256))
+    if hist_hi is None:
+        raise ValueError("hist_hi is required")
+    _need(err_flag, torch.int32, "err_flag")
+    _check(load().eqb_route_hist_fused(_p(z), _p(b), T, E, int(K), _p(mb_offsets), M, _p(topk_idx), _p(tau),
+                                       _p(loads), _p(hist_hi), _p(err_flag), _stream(stream)),
+           "eqb_route_hist_fused")
+    return tau
 
 
 def eqb_margin_hist_pass1(z, tau, hist_hi, err_flag=None, stream=None):
@@ -399,9 +433,12 @@ def eqb_layer_step_noalloc(z, b, K, mb_offsets, loads, b_next, tau=None, topk_id
     """eqb_layer_step without a workspace argument, for callers that cannot
     allocate device memory: the step's scratch is an array inside the
     library (E <= 256).  Calls that overlap on the GPU share that array and
-    race; the first call on a device should come before any stream capture."""
+    race; the first call on a device should come before any stream capture.
+    z (and every other tensor) must be on the current CUDA device: the
+    library looks the scratch array up on that device."""
     T, E = z.shape
     _need(z, torch.bfloat16, "z")
+    _on_current_device(z, "z")
     _need(b, torch.float32, "b", (E,))
     _need(mb_offsets, torch.int64, "mb_offsets")
     M = mb_offsets.numel() - 1

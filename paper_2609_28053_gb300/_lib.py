@@ -19,7 +19,7 @@ EXPORTS = (
     "eqb_layer_step", "eqb_layer_step_noalloc", "eqb_router_route",
     "eqb_router_layer_step", "eqb_maxvio", "gshard_inject_grad",
     "eqb_rank_averaged_bias", "eqb_fixed_hist_bias", "eqb_rank_averaged_workspace_bytes",
-    "eqb_selftest_stalled_wait", "lei_coefficients", "eqb_margin_hist_lei",
+    "eqb_selftest_stalled_wait", "lei_coefficients", "eqb_margin_hist_lei", "eqb_route_hist_fused",
 )
 
 STATUS = {0: "EQB_OK", 1: "EQB_ERR_INVALID_ARG", 2: "EQB_ERR_UNSUPPORTED", 3: "EQB_ERR_CUDA",
@@ -56,6 +56,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
             "lei_inject_grad": [P, P, P, i32, i64, i32, i32, f32, f32, P],
             "lei_coefficients": [P, P, i32, i32, i32, f32, f32, P, P],
             "eqb_margin_hist_lei": [P, P, i64, i32, i32, P, P, P, P, P, P, i32, i64, i64, P],
+            "eqb_route_hist_fused": [P, P, i64, i32, i32, P, i32, P, P, P, P, P, P],
             "eqb_router_logits": [P, P, i64, i32, i32, P, P, P],
             "eqb_maxvio": [P, P, i32, i32, i32, P, P, P],
             "eqb_selftest_stalled_wait": [P, i32, P],

@@ -100,6 +100,22 @@ eqb_status eqb_route_topk(const eqb_bf16* z, const float* b, int64_t T, int32_t 
   return to_status(eqb::launch_hist(h, 1, as_stream(stream)));
 }
 
+eqb_status eqb_route_hist_fused(const eqb_bf16* z, const float* b, int64_t T, int32_t E, int32_t K,
+                                const int64_t* mb_offsets, int32_t M, int32_t* topk_idx, float* tau,
+                                int32_t* loads, int32_t* hist_hi, int32_t* err_flag, void* stream) {
+  eqb_status st = check_shape(T, E, K, true);
+  if (st != EQB_OK) return st;
+  if (!eqb::route_hist_supported(E, K)) return EQB_ERR_UNSUPPORTED;
+  if (!z || !b || !tau || !hist_hi) return EQB_ERR_INVALID_ARG;
+  if (loads && (!mb_offsets || M < 1)) return EQB_ERR_INVALID_ARG;
+  if (!aligned(z, 16) || !aligned(b, 4) || !aligned(tau, 4) || !aligned(topk_idx, 4) ||
+      !aligned(loads, 4) || !aligned(hist_hi, 4) || !aligned(mb_offsets, 8) || !aligned(err_flag, 4))
+    return EQB_ERR_INVALID_ARG;
+  if (T == 0) return EQB_OK;
+  eqb::RouteArgs a{z, b, T, E, K, mb_offsets, M, 0, topk_idx, tau, loads, err_flag};
+  return to_status(eqb::launch_route_hist(a, hist_hi, as_stream(stream)));
+}
+
 eqb_status eqb_margin_hist_pass1(const eqb_bf16* z, const float* tau, int64_t T, int32_t E,
                                  int32_t* hist_hi, int32_t* err_flag, void* stream) {
   eqb_status st = check_shape(T, E, 1, false);

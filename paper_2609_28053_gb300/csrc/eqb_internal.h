@@ -96,8 +96,8 @@ struct GshardArgs {
 constexpr int64_t kLeiCoefCap = 65536;
 
 // The step's scratch, carved from one caller-provided buffer (256-byte
-// aligned pieces): the two [E,256] histograms, u, rho, q_hat and the
-// [M,E] LEI coefficient table.
+// aligned pieces): the two [E,256] histograms (adjacent, cleared together
+// before every step), u, rho, q_hat and the [M,E] LEI coefficient table.
 struct StepWorkspace {
   int32_t* H;
   int32_t* L;
@@ -106,12 +106,23 @@ struct StepWorkspace {
   uint16_t* q;
   float* coef;
 };
-// Carves `base` (or, with base == nullptr, only measures); returns the bytes used.
+constexpr size_t carve_round(size_t n) { return (n + 255) / 256 * 256; }
+constexpr size_t step_workspace_bytes(int E) {
+  return 2 * carve_round(static_cast<size_t>(E) * 1024) + carve_round(static_cast<size_t>(E)) +
+         carve_round(4 * static_cast<size_t>(E)) + carve_round(2 * static_cast<size_t>(E)) +
+         carve_round(4 * static_cast<size_t>(kLeiCoefCap));
+}
+// Carves `base` (or, with base == nullptr, only measures); returns the bytes
+// used, step_workspace_bytes(E) by construction.
 size_t carve_workspace(void* base, int E, StepWorkspace* w);
 
 int launch_route(const RouteArgs& a, cudaStream_t s);
 bool route_wide_supported(int E, int K);
 int launch_route_wide(const RouteArgs& a, cudaStream_t s);
+// Routing and the coarse histogram (hist, [E,256] +=) in one pass over z
+// (route_hist.cu; E = 128 or 256, K + 1 <= 16).
+bool route_hist_supported(int E, int K);
+int launch_route_hist(const RouteArgs& a, int32_t* hist, cudaStream_t s);
 int launch_hist(const HistArgs& a, int pass, cudaStream_t s);
 // A histogram pass (1 or 2) with the injection `ls` streamed beside it.
 int launch_hist_lei(const HistArgs& a, int pass, const LeiStream& ls, cudaStream_t s);

@@ -22,7 +22,7 @@ size_t carve_workspace(void* base, int E, StepWorkspace* w) {
   size_t off = 0;
   auto take = [&](size_t n) {
     uint8_t* p = base ? static_cast<uint8_t*>(base) + off : nullptr;
-    off = (off + n + 255) / 256 * 256;
+    off += carve_round(n);
     return p;
   };
   w->H = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 256 * 4));
@@ -85,9 +85,7 @@ eqb_status check_step(const eqb_bf16* z, const float* b, int64_t T, int32_t E, i
 eqb_status clear(const Workspace& w, int32_t* loads, int32_t E, int32_t M, cudaStream_t s) {
   // H and L are adjacent in the workspace (each E*1 KiB, a multiple of the
   // 256-byte carve alignment): one memset clears both.
-  const size_t hb = static_cast<size_t>(E) * 256 * 4;
-  if (reinterpret_cast<uint8_t*>(w.L) != reinterpret_cast<uint8_t*>(w.H) + hb) return EQB_ERR_CUDA;
-  if (cudaMemsetAsync(w.H, 0, 2 * hb, s) != cudaSuccess ||
+  if (cudaMemsetAsync(w.H, 0, 2 * eqb::carve_round(static_cast<size_t>(E) * 1024), s) != cudaSuccess ||
       cudaMemsetAsync(loads, 0, static_cast<size_t>(M) * E * 4, s) != cudaSuccess)
     return EQB_ERR_CUDA;
   return EQB_OK;

@@ -9,8 +9,10 @@
 // [E,256] histograms, u, rho and q_hat) lives here.
 //
 // The scratch is one file-scope device array sized for the largest supported
-// E (256 experts).  Every GPU that loads this library holds it (about 770
-// KiB) until the process exits.  Host code cannot use the array's name as a
+// E (256 experts): eqb_layer_workspace_bytes(256) = 788,224 bytes (the two
+// [256,256] histograms, u, rho, q_hat and the 65,536-float LEI coefficient
+// table).  Every GPU that loads this library
+// holds it until the process exits.  Host code cannot use the array's name as a
 // device address, so the first call on each device, with that device
 // current, looks the address up once with cudaGetSymbolAddress; make that
 // first call before any stream capture.  All calls on a device share the
@@ -23,10 +25,12 @@
 #include <mutex>
 
 #include "eqb.h"
+#include "eqb_internal.h"
 
 namespace {
 
-constexpr size_t kStaticWorkspaceBytes = 788224;  // eqb_layer_workspace_bytes(256)
+// eqb_layer_workspace_bytes(256): the carve of step.cu measures exactly this.
+constexpr size_t kStaticWorkspaceBytes = eqb::step_workspace_bytes(256);
 static __device__ __align__(256) unsigned char g_step_scratch[kStaticWorkspaceBytes];
 
 constexpr int kMaxDevices = 64;

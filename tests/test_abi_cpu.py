@@ -139,6 +139,26 @@ def test_fused_pass_rejects(lib):
     assert call(T=0, t1=0) == 0
 
 
+def test_route_hist_fused_rejects(lib):
+    """Routing + coarse histogram in one kernel: host-side rejection of bad
+    calls, nothing launched."""
+    f = lib.eqb_route_hist_fused
+
+    def call(T=100, E=256, K=8, M=2, off=FAKE, loads=FAKE, hist=FAKE, tau=FAKE, z=FAKE):
+        return f(z, FAKE, T, E, K, off, M, FAKE, tau, loads, hist, NULL, NULL)
+
+    assert call(E=64) == UNSUPPORTED            # only E = 128 and 256
+    assert call(E=384) == UNSUPPORTED
+    assert call(K=16) == UNSUPPORTED            # K + 1 > 16
+    assert call(hist=NULL) == INVALID
+    assert call(tau=NULL) == INVALID
+    assert call(off=NULL) == INVALID            # loads given without offsets
+    assert call(M=0) == INVALID
+    assert call(z=MISALIGNED) == INVALID
+    assert call(K=0) == INVALID
+    assert call(loads=NULL, off=NULL, M=0, T=0) == 0
+
+
 def test_binding_fails_loudly_without_library(tmp_path):
     from paper_2609_28053_gb300 import _lib
     with pytest.raises(RuntimeError, match="no CPU fallback"):
@@ -184,6 +204,10 @@ def test_layer_step_workspace_size(lib):
     assert lib.eqb_layer_workspace_bytes(256) >= 2 * 256 * 256 * 4 + 256 * 7
     assert lib.eqb_layer_workspace_bytes(256) % 256 == 0
     assert lib.eqb_layer_workspace_bytes(0) == 0
+    # the size the header and the allocation-free entry point state
+    assert lib.eqb_layer_workspace_bytes(256) == 788224
+    src = open(HEADER).read()
+    assert "788,224 bytes" in src
 
 
 def test_layer_step_rejects(lib):
@@ -285,3 +309,24 @@ def test_selftest_rejects(lib):
     assert f(FAKE, 0, NULL) == INVALID
     assert f(FAKE, (1 << 24) + 1, NULL) == INVALID
     assert f(MISALIGNED, 100, NULL) == INVALID
+
+
+def test_noalloc_wrapper_requires_the_current_device(monkeypatch):
+    """eqb_layer_step_noalloc takes its scratch array on the current device,
+    so the binding refuses tensors that live on another one (checked before
+    any call into the library; a stand-in tensor and a stubbed current
+    device, no GPU needed)."""
+    import torch
+    import paper_2609_28053_gb300 as eqb
+
+    class Dev:
+        index = 0
+
+    class Fake:
+        device = Dev()
+
+    monkeypatch.setattr(torch.cuda, "current_device", lambda: 1)
+    with pytest.raises(ValueError, match="current device"):
+        eqb._on_current_device(Fake(), "z")
+    monkeypatch.setattr(torch.cuda, "current_device", lambda: 0)
+    eqb._on_current_device(Fake(), "z")  # same device: accepted
