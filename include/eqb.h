@@ -119,7 +119,9 @@ eqb_status eqb_route_hist_fused(const eqb_bf16 *z, const float *b, int64_t T, in
 
 /* Coarse pass on its own (Algorithm 1 step 1): recomputes the margins from z
  * and tau and accumulates hist_hi[e, kappa(m) >> 8] += 1 over T tokens.
- * Margins of magnitude >= 2^127 or non-finite set EQB_ERR_NONFINITE. */
+ * Margins of magnitude >= 2^127 or non-finite set EQB_ERR_NONFINITE: kappa
+ * gives them the high bytes 0x00 and 0xff, which the method's domain
+ * (|m| < 2^127) leaves out. */
 eqb_status eqb_margin_hist_pass1(const eqb_bf16 *z, const float *tau, int64_t T,
                                  int32_t E, int32_t *hist_hi, int32_t *err_flag,
                                  void *stream);

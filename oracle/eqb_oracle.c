@@ -33,6 +33,10 @@
  *   - kappa maps the bf16 bit pattern x to the 16-bit key
  *       x & 0x8000 ? ~x & 0xffff : x | 0x8000
  *     (so -0 sorts just below +0); a zero quantile is returned as +0;
+ *   - margins must be finite with |m| < 2^127: the high bytes 0x00 and 0xff
+ *     of kappa hold |m| >= 2^127 and the non-finite patterns alike, so the
+ *     coarse pass cannot tell them apart; the quantile and the coarse
+ *     histogram refuse margins there (ORACLE_ERR_NONFINITE);
  *   - the centering mean is an fp64 sum in ascending expert order, divided
  *     by E; b_e = (float)((double)b_hat_e - mean);
  *   - LEI adds eta * rho~_e to every (t, e) of the local batch (selected or
@@ -171,6 +175,10 @@ int oracle_route(const uint16_t *z, const float *b, int64_t T, int32_t E,
   return ORACLE_OK;
 }
 
+/* A margin the method accepts: finite with |m| < 2^127, i.e. a bf16 pattern
+ * whose magnitude bits are below 0x7f00 (kappa high byte 0x01..0xfe). */
+static int margin_in_range(uint16_t m) { return (m & 0x7fffu) < 0x7f00u; }
+
 /* ---- margins and the exact quantile: Eq. (2) ---------------------------- */
 
 /* m_{t,e} = bf16_rne(tau_t - fp32(z_{t,e})) for one expert e, all t. */
@@ -203,7 +211,7 @@ int oracle_quantile(const uint16_t *z, const float *tau, int64_t T, int32_t E,
     if (e < 0 || e >= E) { free(m); return ORACLE_ERR_ARG; }
     oracle_margins(z, tau, T, E, e, m);
     for (int64_t t = 0; t < T; ++t)
-      if (!f32_is_finite(bf16_bits_to_f32(m[t]))) { free(m); return ORACLE_ERR_NONFINITE; }
+      if (!margin_in_range(m[t])) { free(m); return ORACLE_ERR_NONFINITE; }
     qsort(m, (size_t)T, sizeof(uint16_t), cmp_bf16_value);
     uint16_t q = m[r - 1];
     if (q == 0x8000u) q = 0; /* zero is returned as +0 */
@@ -224,6 +232,7 @@ int oracle_hist_hi(const uint16_t *z, const float *tau, int64_t t0, int64_t t1,
   for (int64_t t = t0; t < t1; ++t)
     for (int32_t e = 0; e < E; ++e) {
       uint16_t m = oracle_f32_to_bf16(tau[t] - bf16_bits_to_f32(z[t * E + e]));
+      if (!margin_in_range(m)) return ORACLE_ERR_NONFINITE;
       uint16_t k = oracle_kappa(m);
       H[(int64_t)e * 256 + (k >> 8)] += 1;
     }

@@ -245,6 +245,35 @@ def test_constant_columns_closed_form():
     assert np.allclose(a, eta_f * np.tanh(xi) / xi * rho[None, :], rtol=1e-13, atol=0)
 
 
+def test_margin_domain_boundary():
+    """The margins the method accepts are finite with |m| < 2^127: kappa's
+    high bytes 0x00 and 0xff hold both |m| >= 2^127 and the non-finite
+    patterns.  Constant columns (one cutoff, one margin per expert) put
+    expert 0's margin at the largest bf16 below 2^127 (accepted: its
+    quantile is that value, high byte 0xfe) or at 2^127 itself (refused by
+    the quantile and by the coarse histogram)."""
+    E, K, T = 8, 2, 10
+    base = np.array([0.0, 1.0, 2.0, 3.0, -1.0, -2.0, 0.5, 1.5], np.float32)
+    for z0, ok in [(np.float32(-1.6e38), True), (np.float32(-2.0 ** 127), False)]:
+        cols = base.copy()
+        cols[0] = z0
+        z = np.tile(brute.bf16_bits_from_f32(cols), (T, 1))
+        b = np.zeros(E, np.float32)
+        _, tau, _ = oracle.route(z, b, K)
+        m0 = brute.bf16_bits_from_f32(np.float32(tau[0]) - brute.f32_from_bf16_bits(z[0, :1]))[0]
+        assert (oracle.kappa(int(m0)) >> 8) == (0xFE if ok else 0xFF)
+        r = oracle.target_rank(T, E, K)
+        if ok:
+            q = oracle.quantile(z, tau, r, experts=[0])
+            assert q[0] == m0
+            assert oracle.hist_hi(z, tau)[0, 0xFE] == T
+        else:
+            with pytest.raises(oracle.OracleError):
+                oracle.quantile(z, tau, r, experts=[0])
+            with pytest.raises(oracle.OracleError):
+                oracle.hist_hi(z, tau)
+
+
 # ---------------------------------------------------------------- LEI
 
 def test_lei_invariants():

@@ -386,12 +386,31 @@ def test_nonfinite_bias_sets_flag():
     assert g["err"][0] == 4
 
 
-def test_huge_margin_sets_flag():
+def test_huge_margin_refused_on_both_sides():
+    """A finite margin of magnitude >= 2^127 shares kappa's high byte with
+    the non-finite patterns: the kernels flag it (EQB_ERR_NONFINITE) and the
+    oracle refuses it, the same reading on both sides."""
     z, b = rand_case(100, 64, seed=6)
     z[5, :] = brute.bf16_bits_from_f32(np.float32([3e38]))[0]
     z[5, 0] = brute.bf16_bits_from_f32(np.float32([-3e38]))[0]
     g = gpu_forward(z, b, 8, np.array([0, 100], np.int64))
     assert g["err"][0] == 4
+    _, tau, _ = oracle.route(z, b, 8)
+    with pytest.raises(oracle.OracleError):
+        oracle.quantile(z, tau, oracle.target_rank(100, 64, 8), experts=[0])
+
+
+@pytest.mark.parametrize("E", [64, 128, 256])
+def test_margins_just_below_the_domain_limit(E):
+    """Margins up to the largest bf16 below 2^127 (kappa high byte 0xfe at
+    the top, 0x01 at the bottom) are inside the method's domain: no flag,
+    and everything bit for bit against the oracle."""
+    z, b = rand_case(300, E, seed=8 + E)
+    big = brute.bf16_bits_from_f32(np.float32([1.6e38, -1.6e38]))
+    z[:, 1] = big[1]           # expert 1: margins near +1.6e38
+    z[::3, 2] = big[0]         # expert 2: in the top-K of every third token
+    off = np.array([0, 150, 300], np.int64)
+    assert_forward_equal(gpu_forward(z, b, 8, off), oracle_forward(z, b, 8, off))
 
 
 def test_unreachable_rank_sets_flag():
