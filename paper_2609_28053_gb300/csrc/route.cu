@@ -12,10 +12,10 @@
 // Exact scores are s_e = fp32(z_e) + b_e (fp32, round to nearest even).  The
 // exact work is confined to a small candidate set found with packed bf16x2
 // arithmetic (two experts per instruction):
-//   A. lower bound: L_e = bf16(z_e + RD(b_e)) never exceeds the next bf16
-//      value above s_e, so the (K+1)st largest of G group maxima of L, moved
-//      down two bf16 steps, is <= tau_t (K+1 groups each hold an element at
-//      or above it).  Moving down two more steps gives the filter threshold.
+//   A. lower bound: L_e = bf16(z_e + RD(b_e)) never exceeds the bf16
+//      rounding of s_e, so the (K+1)st largest of G group maxima of L, moved
+//      down one bf16 step, is <= tau_t (K+1 groups each hold an element at
+//      or above it).  Two steps down is the filter threshold.
 //   B. filter: U_e = bf16(z_e + RU(b_e)) >= threshold keeps every e with
 //      s_e >= tau_t (and a few more).  Per 8-expert chunk the passing experts
 //      form an 8-bit mask; chunks with a non-zero mask are listed per lane.
@@ -180,7 +180,15 @@ __global__ void __launch_bounds__(512) route_kernel(RouteArgs a, int64_t tiles_p
     // Near zero, flushing of subnormal bf16 sums could move L by up to
     // 2^-126; lowering theta below that range keeps the bound safe.
     if (fabsf(theta) < 0x1p-124f) theta = -0x1p-124f;
-    const uint32_t thf = bf16_steps_down(__float_as_uint(theta) >> 16, 4u);
+    // Filter threshold: one bf16 step below theta is enough.  KP1 experts have
+    // L_e >= theta, and L_e = RN_bf16(z + RD(b)) <= RN_bf16(s_e) (RN is monotone,
+    // RD(b) <= b, s_e the exact sum), so their exact sums are >= theta - half a
+    // bf16 step and their fp32 scores >= pred(theta): tau >= pred(theta).  An
+    // expert with fp32 score >= tau has an exact sum within half an fp32 step
+    // of it or above, so U_e = RN_bf16(z + RU(b)) >= RN_bf16(s_e) >= pred(theta).
+    // Two steps keep one step of margin (near zero theta was moved below the
+    // range where subnormal flushing could matter).
+    const uint32_t thf = bf16_steps_down(__float_as_uint(theta) >> 16, 2u);
     const uint32_t thf2 = thf | (thf << 16);
 
     // ---- B: per-chunk masks of U >= threshold, chunks with a hit listed

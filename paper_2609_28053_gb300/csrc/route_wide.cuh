@@ -11,9 +11,9 @@
 //      (bf16x2 max/min network) sorts both half-rows' chunk maxima at once,
 //      and the KP1-th largest of all chunk maxima is
 //      min_{i<KP1} max(A[i], B[KP1-1-i]) for the two sorted lists A, B.
-//      KP1 >= K+1 chunks each hold an element with L at or above it, so,
-//      moved down two bf16 steps, it is <= tau_t; two more steps give the
-//      filter threshold.
+//      KP1 >= K+1 chunks each hold an element with L at or above it, so one
+//      bf16 step below it is <= tau_t and bounds every expert that can be
+//      selected; two steps below it is the filter threshold.
 //   B. per-chunk masks of U_e = bf16(z_e + RU(b_e)) >= threshold, every one
 //      of the experts with s_e >= tau_t among them, kept in shared memory,
 //      with the set of non-zero mask words (32 experts each).
@@ -118,7 +118,15 @@ __device__ __forceinline__ void route_row(const uint8_t* rowp, const float* bs, 
   // Near zero, flushing of subnormal bf16 sums could move L by up to
   // 2^-126; lowering theta below that range keeps the bound safe.
   if (fabsf(theta) < 0x1p-124f) theta = -0x1p-124f;
-  const uint32_t thf = bf16_steps_down(__float_as_uint(theta) >> 16, 4u);
+  // Filter threshold: one bf16 step below theta is enough.  KP1 experts have
+  // L_e >= theta, and L_e = RN_bf16(z + RD(b)) <= RN_bf16(s_e) (RN is monotone,
+  // RD(b) <= b, s_e the exact sum), so their exact sums are >= theta - half a
+  // bf16 step and their fp32 scores >= pred(theta): tau >= pred(theta).  An
+  // expert with fp32 score >= tau has an exact sum within half an fp32 step
+  // of it or above, so U_e = RN_bf16(z + RU(b)) >= RN_bf16(s_e) >= pred(theta).
+  // Two steps keep one step of margin (near zero theta was moved below the
+  // range where subnormal flushing could matter).
+  const uint32_t thf = bf16_steps_down(__float_as_uint(theta) >> 16, 2u);
   const uint32_t thf2 = thf | (thf << 16);
 
   // ---- B: per-chunk masks of U >= threshold, stored four to a word (bit

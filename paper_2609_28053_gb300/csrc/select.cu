@@ -19,40 +19,16 @@ namespace eqb {
 
 namespace {
 
-__global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__ hist, int E, int pass,
-                                                     int64_t r, uint8_t* __restrict__ u,
-                                                     int32_t* __restrict__ rho,
-                                                     uint16_t* __restrict__ q_hat, int32_t* err,
-                                                     const int64_t* __restrict__ shard_off, int K) {
-  griddep_wait();
-  const int lane = threadIdx.x & 31;
-  const int e = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-  if (e >= E) return;
-  if (shard_off) {
-    // shard blockIdx.y: its own histogram, outputs and rank ceil(n_p K / E)
-    const int p = blockIdx.y;
-    const int64_t n = shard_off[p + 1] - shard_off[p];
-    hist += (int64_t)p * E * 256;
-    u += (int64_t)p * E;
-    rho += (int64_t)p * E;
-    if (q_hat) q_hat += (int64_t)p * E;
-    if (n <= 0) {
-      if (lane == 0) {
-        if (pass != 2) { u[e] = 0; rho[e] = 0; }
-        else q_hat[e] = 0;
-      }
-      return;
-    }
-    r = (n * K + E - 1) / E;
-  }
-  const int32_t* h = hist + (int64_t)e * 256 + lane * 8;
-  int64_t cnt[8];
+// One warp selects for expert e from its 256 counts, lane j holding bins
+// 8j..8j+7 (cnt): pass 1 writes u[e] and rho[e] for the rank `target`, pass 2
+// writes q_hat[e] from u[e] and the rank target = rho[e].  Flags a count in
+// high-byte bin 0x00 or 0xff (pass 1) and an unreachable rank.
+__device__ __forceinline__ void warp_select(const int64_t (&cnt)[8], int e, int pass, int64_t target,
+                                            uint8_t* __restrict__ u, int32_t* __restrict__ rho,
+                                            uint16_t* __restrict__ q_hat, int32_t* err, int lane) {
   int64_t local = 0;
 #pragma unroll
-  for (int j = 0; j < 8; ++j) {
-    cnt[j] = h[j];
-    local += cnt[j];
-  }
+  for (int j = 0; j < 8; ++j) local += cnt[j];
   int64_t incl = local;
 #pragma unroll
   for (int d = 1; d < 32; d <<= 1) {
@@ -61,7 +37,6 @@ __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__
   }
   const int64_t excl = incl - local;
   const bool first = pass != 2;
-  const int64_t target = first ? r : (int64_t)rho[e];
   const unsigned hit = __ballot_sync(kFull, excl < target && target <= incl);
   if (pass == 1 && ((lane == 0 && cnt[0] != 0) || (lane == 31 && cnt[7] != 0)))
     raise_flag(err, kErrNonfinite);
@@ -94,6 +69,39 @@ __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__
   }
 }
 
+__global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__ hist, int E, int pass,
+                                                     int64_t r, uint8_t* __restrict__ u,
+                                                     int32_t* __restrict__ rho,
+                                                     uint16_t* __restrict__ q_hat, int32_t* err,
+                                                     const int64_t* __restrict__ shard_off, int K) {
+  griddep_wait();
+  const int lane = threadIdx.x & 31;
+  const int e = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+  if (e >= E) return;
+  if (shard_off) {
+    // shard blockIdx.y: its own histogram, outputs and rank ceil(n_p K / E)
+    const int p = blockIdx.y;
+    const int64_t n = shard_off[p + 1] - shard_off[p];
+    hist += (int64_t)p * E * 256;
+    u += (int64_t)p * E;
+    rho += (int64_t)p * E;
+    if (q_hat) q_hat += (int64_t)p * E;
+    if (n <= 0) {
+      if (lane == 0) {
+        if (pass != 2) { u[e] = 0; rho[e] = 0; }
+        else q_hat[e] = 0;
+      }
+      return;
+    }
+    r = (n * K + E - 1) / E;
+  }
+  const int32_t* h = hist + (int64_t)e * 256 + lane * 8;
+  int64_t cnt[8];
+#pragma unroll
+  for (int j = 0; j < 8; ++j) cnt[j] = h[j];
+  warp_select(cnt, e, pass, pass != 2 ? r : (int64_t)rho[e], u, rho, q_hat, err, lane);
+}
+
 // Exponent range of a non-zero bf16 pattern: [ulp exponent, leading-bit exponent].
 __device__ __forceinline__ void bf16_exp_range(uint32_t x, int& lo, int& hi) {
   const int ex = (x >> 7) & 0xff;
@@ -108,15 +116,18 @@ __device__ __forceinline__ void bf16_exp_range(uint32_t x, int& lo, int& hi) {
 // ceil(log2 E) <= 52), any summation order gives the exact sum, so a warp
 // tree reduction reproduces the sequential sum bit for bit.  Otherwise one
 // thread sums in ascending order.
-__global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, float* __restrict__ b_next) {
+// The block computes b_next from q_hat (the threads of the block share the
+// final subtraction; warp 0 forms the mean).
+__device__ __forceinline__ void block_bias_update(const uint16_t* q_hat, int E, float* __restrict__ b_next) {
   __shared__ double mean;
-  griddep_wait();
+  // q_hat may have been written earlier in the same kernel: read it through L2
+
   if (threadIdx.x < 32) {
     const int lane = threadIdx.x;
     double part = 0.0;
     int lo = 1 << 20, hi = -(1 << 20);
     for (int e = lane; e < E; e += 32) {
-      const uint32_t x = q_hat[e];
+      const uint32_t x = __ldcg(q_hat + e);
       if ((x & 0x7fffu) != 0u) {
         int l, h;
         bf16_exp_range(x, l, h);
@@ -139,13 +150,51 @@ __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, fl
     } else {
       sum = 0.0;
       if (lane == 0)
-        for (int e = 0; e < E; ++e) sum = __dadd_rn(sum, (double)bf16_bits_to_f32(q_hat[e]));
+        for (int e = 0; e < E; ++e) sum = __dadd_rn(sum, (double)bf16_bits_to_f32(__ldcg(q_hat + e)));
     }
     if (lane == 0) mean = __ddiv_rn(sum, (double)E);
   }
   __syncthreads();
   for (int e = threadIdx.x; e < E; e += blockDim.x)
-    b_next[e] = __double2float_rn(__dsub_rn((double)bf16_bits_to_f32(q_hat[e]), mean));
+    b_next[e] = __double2float_rn(__dsub_rn((double)bf16_bits_to_f32(__ldcg(q_hat + e)), mean));
+}
+
+
+__global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, float* __restrict__ b_next) {
+  griddep_wait();
+  block_bias_update(q_hat, E, b_next);
+}
+
+// Algorithm 1 steps 5-6 and Eq. (2) in one block: the pass-2 selection of
+// every expert (each warp loads the counts of 4 experts before it scans
+// them), then the bias update.  Same results as select_kernel (pass 2)
+// followed by bias_update_kernel.
+__global__ void __launch_bounds__(1024) select_bias_kernel(const int32_t* __restrict__ hist, int E,
+                                                           const uint8_t* __restrict__ u,
+                                                           int32_t* __restrict__ rho,
+                                                           uint16_t* __restrict__ q_hat, int32_t* err,
+                                                           float* __restrict__ b_next) {
+  constexpr int B = 4;
+  griddep_wait();
+  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
+  for (int e0 = wid; e0 < E; e0 += nw * B) {
+    int4 ca[B], cb[B];
+#pragma unroll
+    for (int k = 0; k < B; ++k) {
+      const int e = e0 + k * nw;
+      const int32_t* h = hist + (int64_t)min(e, E - 1) * 256 + lane * 8;
+      ca[k] = __ldg(reinterpret_cast<const int4*>(h));
+      cb[k] = __ldg(reinterpret_cast<const int4*>(h + 4));
+    }
+#pragma unroll
+    for (int k = 0; k < B; ++k) {
+      const int e = e0 + k * nw;
+      const int64_t cnt[8] = {ca[k].x, ca[k].y, ca[k].z, ca[k].w, cb[k].x, cb[k].y, cb[k].z, cb[k].w};
+      if (e < E) warp_select(cnt, e, 2, (int64_t)rho[e], const_cast<uint8_t*>(u), rho, q_hat, err, lane);
+    }
+  }
+  __syncthreads();  // every q_hat is written
+  block_bias_update(q_hat, E, b_next);
 }
 
 }  // namespace
@@ -166,6 +215,14 @@ int launch_select_sharded(const int32_t* hist, int E, int pass, const int64_t* s
   dim3 grid((E + wpb - 1) / wpb, P);
   return launch_dependent(select_kernel, grid, dim3(wpb * 32), 0, s, hist, E, pass, (int64_t)0, u, rho, q_hat, err,
                           shard_off, K) == cudaSuccess
+             ? kOk
+             : kErrCuda;
+}
+
+int launch_select_bias(const int32_t* hist, int E, const uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err,
+                       float* b_next, cudaStream_t s) {
+  return launch_dependent(select_bias_kernel, dim3(1), dim3(1024), 0, s, hist, E, u, rho, q_hat, err, b_next) ==
+                 cudaSuccess
              ? kOk
              : kErrCuda;
 }

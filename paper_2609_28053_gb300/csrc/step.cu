@@ -112,16 +112,14 @@ eqb_status after_routing(const Workspace& w, const eqb_bf16* z, int64_t T, int32
     if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
     eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};
     if (int rc = eqb::launch_hist_lei(h2, 2, l2, s)) return st(rc);
-    if (int rc = eqb::launch_select(w.L, E, 2, r, w.u, w.rho, w.q, err_flag, s)) return st(rc);
-    if (int rc = eqb::launch_bias_update(w.q, E, b_next, s)) return st(rc);
+    if (int rc = eqb::launch_select_bias(w.L, E, w.u, w.rho, w.q, err_flag, b_next, s)) return st(rc);
     return EQB_OK;
   }
   if (int rc = eqb::launch_hist(h1, 1, s)) return st(rc);
   if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
   eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};
   if (int rc = eqb::launch_hist(h2, 2, s)) return st(rc);
-  if (int rc = eqb::launch_select(w.L, E, 2, r, w.u, w.rho, w.q, err_flag, s)) return st(rc);
-  if (int rc = eqb::launch_bias_update(w.q, E, b_next, s)) return st(rc);
+  if (int rc = eqb::launch_select_bias(w.L, E, w.u, w.rho, w.q, err_flag, b_next, s)) return st(rc);
   if (grad_s) {
     eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
     if (int rc = eqb::launch_lei(la, s)) return st(rc);
