@@ -172,13 +172,19 @@ class Step:
         # entry points.
         self.fused = self.M * E <= 65536
         self.coef = torch.empty((self.M, E), dtype=torch.float32, device=dev)
-        first = ["router_route"] if workload == "router" else ["route_topk"]
-        if self.fused:
-            self.names = first + ["lei_coefficients", "margin_hist_lei_pass1", "select_pass1",
-                                  "margin_hist_lei_pass2", "select_pass2", "bias_update"]
+        if workload == "router":
+            # projection, routing and the coarse histogram in one kernel; the
+            # fine pass carries all of LEI
+            self.names = (["router_route", "lei_coefficients", "select_pass1", "margin_hist_lei_pass2",
+                           "select_pass2", "bias_update"] if self.fused else
+                          ["router_route", "select_pass1", "margin_hist_pass2", "select_pass2", "bias_update",
+                           "lei_inject_grad"])
+        elif self.fused:
+            self.names = ["route_topk", "lei_coefficients", "margin_hist_lei_pass1", "select_pass1",
+                          "margin_hist_lei_pass2", "select_pass2", "bias_update"]
         else:
-            self.names = first + ["margin_hist_pass1", "select_pass1", "margin_hist_pass2",
-                                  "select_pass2", "bias_update", "lei_inject_grad"]
+            self.names = ["route_topk", "margin_hist_pass1", "select_pass1", "margin_hist_pass2",
+                          "select_pass2", "bias_update", "lei_inject_grad"]
 
     def run_step(self, stream):
         """One step through the one-call entry point eqb_layer_step: routing,
@@ -217,10 +223,29 @@ class Step:
         self.loads.zero_()
         if self.workload == "router":
             rec(0, lambda: eqb.eqb_router_route(self.x, self.W, self.b, self.K, self.off, z, self.idx,
-                                                self.tau, self.loads, ws.err, stream))
-        else:
-            rec(0, lambda: eqb.eqb_route_topk(z, self.b, self.K, self.off, self.idx, self.tau,
-                                              self.loads, None, ws.err, stream))
+                                                self.tau, self.loads, ws.err, stream, hist_hi=ws.hist_hi))
+            if world > 1:
+                torch.distributed.all_reduce(ws.hist_hi)
+            k = 1
+            if self.fused:
+                rec(1, lambda: eqb.lei_coefficients(self.loads, self.off, self.K, ETA, C_NORM, self.coef, stream))
+                k = 2
+            rec(k, lambda: eqb.eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream))
+            if self.fused:
+                rec(k + 1, lambda: eqb.eqb_margin_hist_lei(z, self.tau, 2, ws.hist_lo, g, self.coef, self.off, 0,
+                                                           self.T, u=ws.u, stream=stream))
+            else:
+                rec(k + 1, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
+            if world > 1:
+                torch.distributed.all_reduce(ws.hist_lo)
+            rec(k + 2, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err, stream))
+            rec(k + 3, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
+            if not self.fused:
+                rec(k + 4, lambda: eqb.lei_inject_grad(g, self.loads, self.off, self.K, ETA, C_NORM, stream))
+            self.b.copy_(self.b_next)  # b^(q+1) routes step q+1
+            return
+        rec(0, lambda: eqb.eqb_route_topk(z, self.b, self.K, self.off, self.idx, self.tau,
+                                          self.loads, None, ws.err, stream))
         if self.fused:
             th = self.T // 2
             rec(1, lambda: eqb.lei_coefficients(self.loads, self.off, self.K, ETA, C_NORM, self.coef, stream))
@@ -245,23 +270,25 @@ class Step:
         rec(k + 1, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
         if not self.fused:
             rec(6, lambda: eqb.lei_inject_grad(g, self.loads, self.off, self.K, ETA, C_NORM, stream))
-        if self.workload == "router":
-            self.b.copy_(self.b_next)  # b^(q+1) routes step q+1
 
     def launches_per_step(self):
-        """Kernels of this library launched by one timed step (memsets and
-        torch copies excluded): routing, the LEI coefficient table, two
-        histogram passes carrying the injection, two selections and the bias
-        update; without the table, LEI in its own launch instead (for the
-        router workload the routing kernel is the router projection with
-        routing)."""
-        return 7
+        """Kernels of this library launched by one timed one-call step
+        (memsets and torch copies excluded).  Router workload: the projection
+        with routing and the coarse histogram, the LEI coefficient table, two
+        selections (the second with the bias update) and the fine pass
+        carrying LEI: 5.  Otherwise: routing, the coefficient table, two
+        histogram passes carrying the injection, and the two selections (the
+        second with the bias update): 6; without the table, LEI in its own
+        launch instead of the table, still 6."""
+        return 5 if (self.workload == "router" and self.fused) else 6
 
     def algorithmic_bytes(self):
         """Bytes the two-pass method must move per step (see the design notes):
         pass 1 reads z (2TE) and writes idx (4TK) and tau (4T); pass 2 reads z
         (2TE) and tau (4T); LEI reads and writes grad (8TE); the router
-        projection reads x (2Td) and W_r (2Ed) and writes z (2TE).  Per kernel:"""
+        projection reads x (2Td) and W_r (2Ed) and writes z (2TE), and with
+        routing and the coarse histogram in its epilogue leaves only pass 2
+        and LEI to read z.  Per kernel:"""
         T, E, K = self.T, self.E, self.K
         th = T // 2
         d = {"route_topk": 2 * T * E + 4 * T * K + 4 * T,
@@ -270,13 +297,18 @@ class Step:
              "lei_inject_grad": 8 * T * E,
              # the fused passes: the pass's z and tau plus its share of grad
              "margin_hist_lei_pass1": 2 * T * E + 4 * T + 8 * th * E,
-             "margin_hist_lei_pass2": 2 * T * E + 4 * T + 8 * (T - th) * E,
+             "margin_hist_lei_pass2": (2 * T * E + 4 * T + 8 * T * E if self.workload == "router"
+                                       else 2 * T * E + 4 * T + 8 * (T - th) * E),
              "path": 12 * T * E + 8 * T + 4 * T * K}
         if self.workload == "router":
             # the projection reads x and W_r and writes z; routing from its
             # accumulators then adds only idx and tau
             d["router_route"] = 2 * T * self.d + 2 * E * self.d + 2 * T * E + 4 * T * K + 4 * T
-            d["path"] += d["router_route"] - d.pop("route_topk")
+            d.pop("route_topk")
+            # the coarse histogram is counted from the tile just written, so
+            # z is read from memory once more, by the fine pass (which carries
+            # LEI when the coefficient table fits)
+            d["path"] = d["router_route"] + d["margin_hist_pass2"] + d["lei_inject_grad"]
         return d
 
 

@@ -352,17 +352,23 @@ eqb_status eqb_fixed_hist_bias(const eqb_bf16 *z, const float *tau, int64_t T, i
 eqb_status eqb_maxvio(const int32_t *loads, const int64_t *mb_offsets, int32_t M, int32_t E,
                       int32_t K, double *maxvio, double *per_mb, void *stream);
 
-/* Router logits and routing in one kernel: eqb_router_logits followed by
- * eqb_route_topk (without hist_hi), with each token routed straight from the
+/* Router logits, routing and the coarse pass in one kernel: eqb_router_logits
+ * followed by eqb_route_topk, with each token routed straight from the
  * tensor-memory accumulator of its row, so z is written once and not read
- * back.  The paper computes the same two steps one after the other (Sec. 2,
- * Eq. 1, then top-K of s = z + b); fusing them is a property of this library.
- *   x, W_r, z   as in eqb_router_logits; z is still written (the EQB passes
+ * back for routing.  The paper computes the same steps one after the other
+ * (Sec. 2, Eq. 1, then top-K of s = z + b, then Algorithm 1 step 1); fusing
+ * them is a property of this library.
+ *   x, W_r, z   as in eqb_router_logits; z is still written (the fine pass
  *               and LEI read it)
- *   b, K, mb_offsets, M, topk_idx, tau, loads, err_flag
+ *   b, K, mb_offsets, M, topk_idx, tau, loads, hist_hi, err_flag
  *               as in eqb_route_topk: topk_idx [T,K] (nullable), tau [T],
- *               loads [M,E] += (nullable; then mb_offsets may be NULL)
- * Results equal those of the two calls made one after the other on the same
+ *               loads [M,E] += (nullable; then mb_offsets may be NULL),
+ *               hist_hi [E,256] += (nullable): the coarse histogram, counted
+ *               in the same kernel from the rows it just stored (read back
+ *               from L2) when no block of the kernel routes more than 65,535
+ *               tokens (T <= 65,535 x the SM count, rounded down to 128-row
+ *               tiles), else by the coarse pass over z after it
+ * Results equal those of the calls made one after the other on the same
  * inputs, bit for bit.  err_flag: EQB_ERR_NONFINITE as in eqb_route_topk,
  * EQB_ERR_CUDA as in eqb_router_logits.
  * Supported: E in {64, 128}, 1 <= K <= 8, K < E, d a positive multiple of
@@ -371,13 +377,15 @@ eqb_status eqb_maxvio(const int32_t *loads, const int64_t *mb_offsets, int32_t M
 eqb_status eqb_router_route(const eqb_bf16 *x, const eqb_bf16 *W_r, int64_t T, int32_t d,
                             int32_t E, int32_t K, const float *b, const int64_t *mb_offsets,
                             int32_t M, eqb_bf16 *z, int32_t *topk_idx, float *tau,
-                            int32_t *loads, int32_t *err_flag, void *stream);
+                            int32_t *loads, int32_t *hist_hi, int32_t *err_flag, void *stream);
 
 /* The routing-balance step of one layer from the router input: the router
  * projection z = bf16(x W_r^T) (Sec. 2, Eq. 1) followed by everything
- * eqb_layer_step does.  For E in {64, 128} and K <= 8 the projection and the
- * routing run as one kernel (eqb_router_route); otherwise as
- * eqb_router_logits then eqb_route_topk.  The other steps are those of
+ * eqb_layer_step does.  For E in {64, 128} and K <= 8 the projection, the
+ * routing and the coarse histogram run as one kernel (eqb_router_route with
+ * hist_hi), and the fine pass then streams all of LEI (when M * E <=
+ * 65,536); otherwise eqb_router_logits then eqb_route_topk and the schedule
+ * of eqb_layer_step.  The other steps are those of
  * eqb_layer_step, and so are the arguments from b on; z is an output here
  * (device bf16 [T,E], 16-byte aligned).
  *   x, W_r, d   as in eqb_router_logits.

@@ -229,9 +229,10 @@ def eqb_router_logits(x, W_r, z=None, err_flag=None, stream=None):
 
 
 def eqb_router_route(x, W_r, b, K, mb_offsets=None, z=None, topk_idx=None, tau=None, loads=None,
-                     err_flag=None, stream=None):
+                     err_flag=None, stream=None, hist_hi=None):
     """Router logits and routing in one kernel (see eqb.h): z = bf16(x W_r^T)
     and, from the same accumulators, eqb_route_topk's topk_idx, tau and loads
+    (accumulated into); with hist_hi [E,256] also the coarse histogram
     (accumulated into).  E in {64, 128}, K <= 8.  Returns (z, topk_idx, tau)."""
     T, d = x.shape
     E = W_r.shape[0]
@@ -250,9 +251,10 @@ def eqb_router_route(x, W_r, b, K, mb_offsets=None, z=None, topk_idx=None, tau=N
         _need(mb_offsets, torch.int64, "mb_offsets")
         M = mb_offsets.numel() - 1
     _need(loads, torch.int32, "loads", (M, E) if loads is not None else None)
+    _need(hist_hi, torch.int32, "hist_hi", (E, 256) if hist_hi is not None else None)
     _need(err_flag, torch.int32, "err_flag")
     _check(load().eqb_router_route(_p(x), _p(W_r), T, d, E, K, _p(b), _p(mb_offsets), M, _p(z),
-                                   _p(topk_idx), _p(tau), _p(loads), _p(err_flag), _stream(stream)),
+                                   _p(topk_idx), _p(tau), _p(loads), _p(hist_hi), _p(err_flag), _stream(stream)),
            "eqb_router_route")
     return z, topk_idx, tau
 

@@ -63,7 +63,7 @@ def load(path: str | None = None) -> ctypes.CDLL:
             "gshard_inject_grad": [P, P, P, P, i32, i64, i32, i32, f32, P],
             "eqb_rank_averaged_bias": [P, P, i64, i32, i32, P, i32, P, P, P, ctypes.c_size_t, P, P],
             "eqb_fixed_hist_bias": [P, P, i64, i32, i32, f32, f32, P, P, P, ctypes.c_size_t, P, P],
-            "eqb_router_route": [P, P, i64, i32, i32, i32, P, P, i32, P, P, P, P, P, P],
+            "eqb_router_route": [P, P, i64, i32, i32, i32, P, P, i32, P, P, P, P, P, P, P],
             "eqb_router_layer_step": [P, P, i64, i32, i32, i32, P, P, P, i32, i64, P, P, P, P, P, P,
                                       f32, f32, P, ctypes.c_size_t, P, P],
             "eqb_layer_step": [P, P, i64, i32, i32, P, P, i32, i64, P, P, P, P, P, f32, f32, P,

@@ -215,18 +215,20 @@ eqb_status eqb_router_logits(const eqb_bf16* x, const eqb_bf16* W_r, int64_t T, 
 
 eqb_status eqb_router_route(const eqb_bf16* x, const eqb_bf16* W_r, int64_t T, int32_t d, int32_t E,
                             int32_t K, const float* b, const int64_t* mb_offsets, int32_t M, eqb_bf16* z,
-                            int32_t* topk_idx, float* tau, int32_t* loads, int32_t* err_flag, void* stream) {
+                            int32_t* topk_idx, float* tau, int32_t* loads, int32_t* hist_hi, int32_t* err_flag,
+                            void* stream) {
   if (T < 0 || d < 1 || E < 2 || K < 1 || K >= E) return EQB_ERR_INVALID_ARG;
   if ((d % 64) != 0 || (E != 64 && E != 128) || K > 8) return EQB_ERR_UNSUPPORTED;
   if (T > (int64_t(1) << 31) - (int64_t(1) << 24)) return EQB_ERR_UNSUPPORTED;
   if (!x || !W_r || !z || !b || !tau) return EQB_ERR_INVALID_ARG;
   if (loads && (!mb_offsets || M < 1)) return EQB_ERR_INVALID_ARG;
   if (!aligned(x, 16) || !aligned(W_r, 16) || !aligned(z, 16) || !aligned(b, 4) || !aligned(tau, 4) ||
-      !aligned(topk_idx, 4) || !aligned(loads, 4) || !aligned(mb_offsets, 8) || !aligned(err_flag, 4))
+      !aligned(topk_idx, 4) || !aligned(loads, 4) || !aligned(hist_hi, 4) || !aligned(mb_offsets, 8) ||
+      !aligned(err_flag, 4))
     return EQB_ERR_INVALID_ARG;
   if (T == 0) return EQB_OK;
   return to_status(eqb::launch_router_route(x, W_r, T, d, E, K, b, mb_offsets, M, z, topk_idx, tau, loads,
-                                            err_flag, as_stream(stream)));
+                                            hist_hi, err_flag, as_stream(stream)));
 }
 
 eqb_status eqb_maxvio(const int32_t* loads, const int64_t* mb_offsets, int32_t M, int32_t E, int32_t K,

@@ -148,8 +148,12 @@ int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, i
 int launch_gshard(const GshardArgs& a, cudaStream_t s);
 int launch_maxvio(const int32_t* loads, const int64_t* off, int M, int E, int K, double* out, double* per_mb,
                   cudaStream_t s);
+// The router projection routing each token from its accumulators (E = 64 or
+// 128, K <= 8); with hist (nullable) also the coarse histogram ([E,256] +=),
+// counted in the epilogue when no block routes more than 65,535 tokens, else
+// by the coarse pass over z after it.
 int launch_router_route(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, int K, const float* b,
                         const int64_t* off, int M, uint16_t* z, int32_t* idx, float* tau, int32_t* loads,
-                        int32_t* err, cudaStream_t s);
+                        int32_t* hist, int32_t* err, cudaStream_t s);
 
 }  // namespace eqb

@@ -9,21 +9,10 @@
 // taking the 8 experts of chunk c of each token.  z is read from DRAM once
 // for both, where the separate kernels read it twice.
 //
-// Coarse bins.  The 256 bins of all E experts would not leave room for the
-// routing tiles, so the block keeps 16-bit counters (two experts per word)
-// only for the bins that hold practically every margin: |m| in
-// [2^-15, 2^17), both signs (32 of the 256 high bytes).  A margin outside
-// that window is added straight to the global histogram.  In terms of the
-// internal key hk = kappa(m) >> 8 ^ 0x80, sl = (hk - 56) mod 256 lies in
-// [0, 16) for m >= 0 and in [128, 144) for m < 0 inside the window, and the
-// counter of pair row r and sl is word 289 (r >> 3) + 16 pos(r) + sl with
-// pos(r) = ((r & 3) << 1) | ((r >> 2) & 1): the two 16-word segments of a
-// row are 128 words apart, eight rows fill 256 words, and the (r >> 3)
-// skew puts equal bins of the 32 lanes of a warp in 32 banks.  High byte 0
-// (+0, subnormal and the smallest normal positive margins: the cutoff
-// expert's own margin whenever its bias is 0) has a counter of its own per
-// row in the 33 spare words after each eight rows.  Counters are added into
-// H at least every 65,535 tokens per block and at the end.
+// Coarse bins: the window of 16-bit shared-memory counters of
+// coarse_window.cuh (the 256 bins of all E experts would not leave room for
+// the routing tiles).  Counters are added into H at least every 65,535
+// tokens per block and at the end.
 //
 // On GB300 this kernel is slower than routing and the coarse pass as two
 // kernels: both are bound by instruction issue (ALU pipe), not by DRAM, so
@@ -31,14 +20,12 @@
 // routing for the same ALU pipe at a third of the coarse pass's occupancy.
 // The one-call step therefore uses the two kernels; this one is the
 // one-read variant (eqb_route_hist_fused).
+#include "coarse_window.cuh"
 #include "route_wide.cuh"
 
 namespace eqb {
 
 namespace {
-
-constexpr uint32_t kWinBias = 0x00c800c8u;  // -56 mod 256 in both 16-bit lanes
-constexpr int kWinLo = 56;
 
 template <int E>
 struct FusedLayout {
@@ -48,7 +35,7 @@ struct FusedLayout {
   static constexpr int ENT = W::ENT;
   static constexpr int WL = W::WL;
   static constexpr int WARP = W::WARP;          // tile, masks, load counters, mbarrier
-  static constexpr int BINW = (E / 16) * 289;   // windowed bin words
+  static constexpr int BINW = coarse_window_words(E);
   static constexpr int OFF_RD = 4 * E;
   static constexpr int OFF_RU = OFF_RD + 2 * E;
   static constexpr int OFF_BINS = OFF_RU + 2 * E;
@@ -103,11 +90,8 @@ __global__ void __launch_bounds__(32 * NW, 1)
 
   // ---- this lane's counters while counting: chunk cc of token slot ctok
   const int cc = lane % LPT, ctok = lane / LPT;
-  uint32_t cbase[4];
-#pragma unroll
-  for (int p = 0; p < 4; ++p)
-    cbase[p] = saddr(bins) + 4u * static_cast<uint32_t>(289 * (cc >> 1) + 16 * ((p << 1) | (cc & 1)));
-  const uint32_t zbase = saddr(bins) + 4u * static_cast<uint32_t>(289 * (cc >> 1) + 256 + 4 * (cc & 1));
+  uint32_t cbase[4], zbase;
+  coarse_window_bases(saddr(bins), cc, cbase, zbase);
 
   // ---- the warp's contiguous tile range
   const int64_t ntiles = (T + 31) >> 5;
@@ -147,62 +131,6 @@ __global__ void __launch_bounds__(32 * NW, 1)
     __syncwarp();
   };
 
-  // ---- counting one token's chunk (8 experts, 4 packed words) of the tile
-  auto count = [&](const uint4& w4, float tv) {
-    const uint32_t zw[4] = {w4.x, w4.y, w4.z, w4.w};
-    const uint64_t tt = f32x2_splat(tv);
-#pragma unroll
-    for (int p = 0; p < 4; ++p) {
-      const uint32_t m = margins_bf16x2(tt, zw[p]);
-      const uint32_t k = kappa2_internal(m);
-      const uint32_t y = prmt(k, 0u, 0x4341u) + kWinBias;  // (hk - 56) per 16-bit lane (+ a carry bit)
-      if ((y & 0x00700070u) == 0u) {
-        const uint32_t s0 = y & 0x8fu, s1 = (y >> 16) & 0x8fu;
-        if (s0 == s1) {
-          red_shared_add(cbase[p] + 4u * s0, 0x10001u);
-        } else {
-          red_shared_add(cbase[p] + 4u * s0, 1u);
-          red_shared_add(cbase[p] + 4u * s1, 0x10000u);
-        }
-      } else {
-#pragma unroll
-        for (int h = 0; h < 2; ++h) {
-          const uint32_t sh = (y >> (16 * h)) & 0xffu;
-          const uint32_t hk = (k >> (8 + 16 * h)) & 0xffu;  // internal high byte
-          if ((sh & 0x70u) == 0u) {
-            red_shared_add(cbase[p] + 4u * sh, h ? 0x10000u : 1u);
-          } else if (hk == 0u) {
-            red_shared_add(zbase + 4u * p, h ? 0x10000u : 1u);
-          } else {
-            const uint32_t hb = hk ^ 0x80u;  // true high byte
-            const int e = cc * 8 + 2 * p + h;
-            atomicAdd(hist + (int64_t)e * 256 + hb, 1);
-            if (hb == 0u || hb == 255u) raise_flag(a.err, kErrNonfinite);
-          }
-        }
-      }
-    }
-  };
-  auto flush_bins = [&]() {
-    for (int w = threadIdx.x; w < L::BINW; w += blockDim.x) {
-      const uint32_t v = bins[w];
-      if (!v) continue;
-      bins[w] = 0u;
-      const int blk = w / 289, o = w - 289 * blk;
-      int e, hb;
-      if (o < 256) {
-        const int pos = (o & 127) >> 4, sl = (o & 15) | (o & 128);
-        e = 2 * (8 * blk + (((pos & 1) << 2) | (pos >> 1)));
-        hb = ((sl + kWinLo) & 0xff) ^ 0x80;
-      } else {
-        e = 2 * (8 * blk + (o - 256));  // the row's high-byte-0 counter
-        hb = 0x80;
-      }
-      if (v & 0xffffu) atomicAdd(hist + (int64_t)e * 256 + hb, static_cast<int>(v & 0xffffu));
-      if (v >> 16) atomicAdd(hist + (int64_t)(e + 1) * 256 + hb, static_cast<int>(v >> 16));
-    }
-  };
-
   bool alive = true;  // false once a copy ran out of time
   uint32_t phase = 0;
   if (tb < te) {
@@ -237,7 +165,8 @@ __global__ void __launch_bounds__(32 * NW, 1)
       for (int j0 = 0; j0 < 32; j0 += TPS) {
         const int j = j0 + ctok;
         const float tv = __shfl_sync(kFull, tau_t, j);
-        if ((tl << 5) + j < T) count(lds128(tile + j * L::RS + 16 * cc), tv);
+        if ((tl << 5) + j < T)
+          coarse_window_count<false>(lds128(tile + j * L::RS + 16 * cc), tv, cbase, zbase, cc, hist, a.err);
       }
       __syncwarp();  // every lane is done with the tile
       if (tl + 1 < te) {
@@ -287,13 +216,13 @@ __global__ void __launch_bounds__(32 * NW, 1)
     }
     if ((k + 1) % kFlushTiles == 0 && k + 1 < tiles_per_warp) {
       __syncthreads();
-      flush_bins();
+      coarse_window_flush(bins, L::BINW, hist, threadIdx.x, blockDim.x);
       __syncthreads();
     }
   }
   if (a.loads) flush_loads();
   __syncthreads();
-  flush_bins();
+  coarse_window_flush(bins, L::BINW, hist, threadIdx.x, blockDim.x);
 }
 
 template <int E, int KP1>

@@ -10,7 +10,13 @@
 //               thread; tcgen05.commit frees each stage and, at the end of a
 //               tile, signals the accumulator as full;
 //   warps 2..5  epilogue: tcgen05.ld of the accumulator (warp w reads TMEM
-//               lanes 32*(w%4) ..+31 = its 32 rows), round to bf16, store z.
+//               lanes 32*(w%4) ..+31 = its 32 rows), round to bf16, store z;
+//               with routing (E = 64, 128) each lane also routes its token
+//               from the accumulator, and with the coarse histogram the warp
+//               then recounts its 32 stored rows (read back from L2, lane c
+//               taking experts 8c..8c+7 of a token) into the window bins of
+//               coarse_window.cuh (Algorithm 1 step 1), so the coarse pass
+//               does not read z again.
 // Two accumulators (2 x E fp32 columns of TMEM) alternate, so the epilogue
 // of one tile overlaps the MMAs of the next.
 //
@@ -20,6 +26,7 @@
 // reports EQB_ERR_CUDA through the error word.
 #include <cuda.h>
 
+#include "coarse_window.cuh"
 #include "eqb_device.cuh"
 
 namespace eqb {
@@ -146,6 +153,7 @@ struct GemmArgs {
   int32_t* idx;
   float* tau;
   int32_t* loads;
+  int32_t* hist;  // the coarse histogram [E,256] (+=), HIST kernels only
 };
 
 // Routing state of one token: the running top-(K+1) of s = fp32(z) + b.
@@ -171,13 +179,20 @@ __device__ __forceinline__ void route_chunk(TopState<KP1>& st, const uint32_t (&
   }
 }
 
-// tau, the top-K list and the loads of one routed token.
-template <int EC, int KP1>
-__device__ __forceinline__ void route_outputs(const TopState<KP1>& st, int row, const GemmArgs& a) {
-  const int K = a.K;
+// The cutoff tau_t = v[K] of a routed token.
+template <int KP1>
+__device__ __forceinline__ float top_tau(const TopState<KP1>& st, int K) {
   float tau_t = st.v[0];
 #pragma unroll
   for (int j = 1; j < KP1; ++j) tau_t = (j == K) ? st.v[j] : tau_t;
+  return tau_t;
+}
+
+// tau and the top-K list of one routed token.
+template <int EC, int KP1>
+__device__ __forceinline__ void route_outputs(const TopState<KP1>& st, int row, const GemmArgs& a) {
+  const int K = a.K;
+  const float tau_t = top_tau<KP1>(st, K);
   a.tau[row] = tau_t;
   if (st.nan || !isfinite(tau_t)) raise_flag(a.err, kErrNonfinite);
   if (a.idx) {
@@ -247,8 +262,11 @@ __device__ __forceinline__ void count_loads(WarpLoads<EC>& wl, const TopState<KP
 }
 
 // EC = 0: the plain GEMM for any supported N.  EC > 0: N = EC and the
-// epilogue also routes each token (K + 1 <= KP1).
-template <int EC, int KP1>
+// epilogue also routes each token (K + 1 <= KP1).  HIST: the epilogue also
+// counts the coarse histogram into a.hist (launched only when no block
+// counts more than 65,535 tokens, so the 16-bit window counters are added
+// into H once, at the end).
+template <int EC, int KP1, bool HIST>
 __global__ void __launch_bounds__(192, 1)
     router_gemm_kernel(const __grid_constant__ CUtensorMap tmx, const __grid_constant__ CUtensorMap tmw,
                        GemmArgs a) {
@@ -274,6 +292,8 @@ __global__ void __launch_bounds__(192, 1)
   // routing only: b (EC floats), then 4 warps x EC/2 packed load counters
   float* bsm = reinterpret_cast<float*>(tmem_holder + 4);
   uint32_t* lcnt = reinterpret_cast<uint32_t*>(bsm + EC);
+  uint32_t* bins = lcnt + 2 * EC;  // coarse window counters (HIST)
+  constexpr int kBinWords = HIST ? coarse_window_words(EC) : 0;
 
   const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
   if (EC > 0) {
@@ -283,6 +303,7 @@ __global__ void __launch_bounds__(192, 1)
       if (!isfinite(bv)) raise_flag(err, kErrNonfinite);
     }
     for (int w = threadIdx.x; w < 2 * EC; w += blockDim.x) lcnt[w] = 0;
+    for (int w = threadIdx.x; w < kBinWords; w += blockDim.x) bins[w] = 0u;
   }
   const int ntiles = (T + kBM - 1) / kBM;
   const int KB = d / kBK;
@@ -367,6 +388,11 @@ __global__ void __launch_bounds__(192, 1)
     const int q = warp & 3;  // TMEM lane quarter accessible to this warp
     const uint32_t lane_base = static_cast<uint32_t>(q * 32) << 16;
     WarpLoads<EC> wl{lcnt + (warp - 2) * (EC / 2), -1, 0};
+    // coarse counting: lane cc of token slot ctok takes experts 8cc..8cc+7
+    constexpr int LPT = EC > 0 ? EC / 8 : 1, TPS = 32 / LPT;
+    const int cc = lane % LPT, ctok = lane / LPT;
+    uint32_t cbase[4], zbase = 0;
+    if constexpr (HIST) coarse_window_bases(smem_u32(bins), cc, cbase, zbase);
     int it = 0;
     for (int tile = blockIdx.x; tile < ntiles; tile += gridDim.x, ++it) {
       const int buf = it & 1;
@@ -421,6 +447,34 @@ __global__ void __launch_bounds__(192, 1)
         mbar_arrive(acce(buf));
         if (row < T) route_outputs<EC, KP1>(st, row, a);
         if (a.loads) count_loads<EC, KP1>(wl, st, row < T, row, a, lane);
+        if constexpr (HIST) {
+          // the coarse histogram of the warp's 32 rows, read back from L2
+          // (every lane's z stores of this tile are ordered before the loads)
+          // Four rows a batch, their loads issued before the batch's counts
+          // (the shared-memory adds are ordered against memory); the loop
+          // over batches stays rolled to keep the epilogue's code small.
+          __syncwarp();
+          const float tau_t = top_tau<KP1>(st, a.K);
+          const int row0 = tile * kBM + q * 32;
+          constexpr int NJ = 32 / TPS, NB = 4;
+#pragma unroll 1
+          for (int i0 = 0; i0 < NJ; i0 += NB) {
+            uint4 w4[NB];
+#pragma unroll
+            for (int i = 0; i < NB; ++i) {
+              const int j = (i0 + i) * TPS + ctok;
+              w4[i] = row0 + j < T
+                          ? __ldcg(reinterpret_cast<const uint4*>(z + static_cast<size_t>(row0 + j) * EC + 8 * cc))
+                          : make_uint4(0u, 0u, 0u, 0u);
+            }
+#pragma unroll
+            for (int i = 0; i < NB; ++i) {
+              const int j = (i0 + i) * TPS + ctok;
+              const float tv = __shfl_sync(0xffffffffu, tau_t, j);
+              if (row0 + j < T) coarse_window_count<true>(w4[i], tv, cbase, zbase, cc, a.hist, err);
+            }
+          }
+        }
       }
     }
     if constexpr (EC > 0) {
@@ -429,6 +483,7 @@ __global__ void __launch_bounds__(192, 1)
   }
   tc_fence_before();
   __syncthreads();
+  if constexpr (HIST) coarse_window_flush(bins, kBinWords, a.hist, threadIdx.x, blockDim.x);
   if (warp == 1) {
     tc_fence_after();
     asm volatile("tcgen05.dealloc.cta_group::1.sync.aligned.b32 %0, %1;" ::"r"(tmem), "r"(kTmemCols)
@@ -473,7 +528,7 @@ bool make_map(CUtensorMap* m, const void* ptr, uint64_t rows, uint64_t cols, uin
 
 namespace {
 
-template <int EC, int KP1>
+template <int EC, int KP1, bool HIST>
 int launch_gemm(const uint16_t* x, const uint16_t* W, GemmArgs a, cudaStream_t s) {
   DeviceInfo di;
   if (int rc = device_info(&di)) return rc;
@@ -484,7 +539,7 @@ int launch_gemm(const uint16_t* x, const uint16_t* W, GemmArgs a, cudaStream_t s
   const int stage_bytes = (kBM + a.N) * kBK * 2;
   // alignment slack, 2S+5 mbarriers (S <= 8), TMEM address + abort flag, b,
   // the epilogue warps' load counters
-  const int extra = 1024 + 8 * (2 * 8 + 5) + 16 + 4 * EC + 8 * EC;
+  const int extra = 1024 + 8 * (2 * 8 + 5) + 16 + 4 * EC + 8 * EC + (HIST ? 4 * coarse_window_words(EC) : 0);
   int S = (di.max_smem_optin - extra) / stage_bytes;
   if (S > 8) S = 8;
   if (S < 2) return kErrUnsupported;
@@ -492,10 +547,10 @@ int launch_gemm(const uint16_t* x, const uint16_t* W, GemmArgs a, cudaStream_t s
   const int smem = S * stage_bytes + extra;
   const int ntiles = (a.T + kBM - 1) / kBM;
   const int grid = ntiles < di.sm_count ? ntiles : di.sm_count;
-  if (cudaFuncSetAttribute(router_gemm_kernel<EC, KP1>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
+  if (cudaFuncSetAttribute(router_gemm_kernel<EC, KP1, HIST>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem) !=
       cudaSuccess)
     return kErrCuda;
-  router_gemm_kernel<EC, KP1><<<grid, 192, smem, s>>>(tmx, tmw, a);
+  router_gemm_kernel<EC, KP1, HIST><<<grid, 192, smem, s>>>(tmx, tmw, a);
   return cudaGetLastError() == cudaSuccess ? kOk : kErrCuda;
 }
 
@@ -503,17 +558,41 @@ int launch_gemm(const uint16_t* x, const uint16_t* W, GemmArgs a, cudaStream_t s
 
 int launch_router_gemm(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, uint16_t* z,
                        int32_t* err, cudaStream_t s) {
-  GemmArgs a{z, static_cast<int>(T), d, E, 0, err, nullptr, 0, nullptr, 0, nullptr, nullptr, nullptr};
-  return launch_gemm<0, 1>(x, W, a, s);
+  GemmArgs a{z, static_cast<int>(T), d, E, 0, err, nullptr, 0, nullptr, 0, nullptr, nullptr, nullptr, nullptr};
+  return launch_gemm<0, 1, false>(x, W, a, s);
 }
+
+namespace {
+
+template <int EC, bool HIST>
+int launch_route_ec(const uint16_t* x, const uint16_t* W, const GemmArgs& a, cudaStream_t s) {
+  return a.K + 1 <= 3 ? launch_gemm<EC, 3, HIST>(x, W, a, s) : launch_gemm<EC, 9, HIST>(x, W, a, s);
+}
+
+}  // namespace
 
 int launch_router_route(const uint16_t* x, const uint16_t* W, int64_t T, int d, int E, int K, const float* b,
                         const int64_t* off, int M, uint16_t* z, int32_t* idx, float* tau, int32_t* loads,
-                        int32_t* err, cudaStream_t s) {
-  GemmArgs a{z, static_cast<int>(T), d, E, 0, err, b, K, off, M, idx, tau, loads};
-  if (E == 64) return K + 1 <= 3 ? launch_gemm<64, 3>(x, W, a, s) : launch_gemm<64, 9>(x, W, a, s);
-  if (E == 128) return K + 1 <= 3 ? launch_gemm<128, 3>(x, W, a, s) : launch_gemm<128, 9>(x, W, a, s);
-  return kErrUnsupported;
+                        int32_t* hist, int32_t* err, cudaStream_t s) {
+  GemmArgs a{z, static_cast<int>(T), d, E, 0, err, b, K, off, M, idx, tau, loads, hist};
+  if (E != 64 && E != 128) return kErrUnsupported;
+  bool in_epilogue = false;
+  if (hist) {
+    // the epilogue's 16-bit window counters are added into H once, at the
+    // end: only while no block counts more than 65,535 tokens
+    DeviceInfo di;
+    if (int rc = device_info(&di)) return rc;
+    const int64_t ntiles = (T + kBM - 1) / kBM;
+    const int64_t grid = ntiles < di.sm_count ? ntiles : di.sm_count;
+    in_epilogue = (ntiles + grid - 1) / grid * kBM <= 65535;
+  }
+  int rc;
+  if (E == 64) rc = in_epilogue ? launch_route_ec<64, true>(x, W, a, s) : launch_route_ec<64, false>(x, W, a, s);
+  else rc = in_epilogue ? launch_route_ec<128, true>(x, W, a, s) : launch_route_ec<128, false>(x, W, a, s);
+  if (rc || !hist || in_epilogue) return rc;
+  // larger T: the coarse pass as its own kernel over the z just written
+  HistArgs h{z, tau, T, E, nullptr, hist, err};
+  return launch_hist(h, 1, s);
 }
 
 }  // namespace eqb

@@ -9,7 +9,9 @@
 // stream the injection, half of the tokens each; otherwise it runs last.
 // All on one stream.
 // eqb_router_layer_step starts one step earlier, at the router projection
-// (Eq. 1), and routes from the projection's accumulators where it can.
+// (Eq. 1), and routes from the projection's accumulators where it can; that
+// kernel also counts the coarse histogram, so the fine pass alone reads z
+// again and carries all of LEI.
 #include <cuda_runtime.h>
 #include <stdint.h>
 
@@ -127,6 +129,34 @@ eqb_status after_routing(const Workspace& w, const eqb_bf16* z, int64_t T, int32
   return EQB_OK;
 }
 
+// Everything after routing when the coarse histogram H was already counted
+// (the router projection's epilogue): selection, the fine pass, selection
+// and the bias update, with LEI streamed entirely by the fine pass when the
+// [M,E] coefficient table fits the workspace, else run last.
+eqb_status after_coarse(const Workspace& w, const eqb_bf16* z, int64_t T, int32_t E, int32_t K,
+                        const int64_t* mb_offsets, int32_t M, int64_t r, const float* tau, const int32_t* loads,
+                        float* b_next, float* grad_s, float eta, float c, int32_t* err_flag, cudaStream_t s) {
+  const bool lei = grad_s && static_cast<int64_t>(M) * E <= eqb::kLeiCoefCap;
+  if (lei) {
+    eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
+    if (int rc = eqb::launch_lei_coef(la, w.coef, s)) return st(rc);
+  }
+  if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
+  eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};
+  if (lei) {
+    eqb::LeiStream l2{grad_s, w.coef, mb_offsets, M, 0, T};
+    if (int rc = eqb::launch_hist_lei(h2, 2, l2, s)) return st(rc);
+  } else {
+    if (int rc = eqb::launch_hist(h2, 2, s)) return st(rc);
+  }
+  if (int rc = eqb::launch_select_bias(w.L, E, w.u, w.rho, w.q, err_flag, b_next, s)) return st(rc);
+  if (grad_s && !lei) {
+    eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
+    if (int rc = eqb::launch_lei(la, s)) return st(rc);
+  }
+  return EQB_OK;
+}
+
 }  // namespace
 
 extern "C" {
@@ -165,9 +195,11 @@ eqb_status eqb_router_layer_step(const eqb_bf16* x, const eqb_bf16* W_r, int64_t
   cudaStream_t s = reinterpret_cast<cudaStream_t>(stream);
   if ((rs = clear(w, loads, E, M, s)) != EQB_OK) return rs;
   if ((E == 64 || E == 128) && K <= 8) {
-    if (int rc = eqb::launch_router_route(x, W_r, T, d, E, K, b, mb_offsets, M, z, topk_idx, tau, loads,
+    // projection, routing and the coarse histogram in one kernel
+    if (int rc = eqb::launch_router_route(x, W_r, T, d, E, K, b, mb_offsets, M, z, topk_idx, tau, loads, w.H,
                                           err_flag, s))
       return st(rc);
+    return after_coarse(w, z, T, E, K, mb_offsets, M, r, tau, loads, b_next, grad_s, eta, c, err_flag, s);
   } else {
     if (int rc = eqb::launch_router_gemm(x, W_r, T, d, E, z, err_flag, s)) return st(rc);
     eqb::RouteArgs ra{z, b, T, E, K, mb_offsets, M, 0, topk_idx, tau, loads, err_flag};

@@ -180,8 +180,8 @@ def test_router_route_rejects(lib):
     f = lib.eqb_router_route
 
     def call(x=FAKE, T=10, d=4096, E=128, K=8, b=FAKE, off=FAKE, M=1, z=FAKE, idx=FAKE, tau=FAKE,
-             loads=FAKE):
-        return f(x, FAKE, T, d, E, K, b, off, M, z, idx, tau, loads, NULL, NULL)
+             loads=FAKE, hist=NULL):
+        return f(x, FAKE, T, d, E, K, b, off, M, z, idx, tau, loads, hist, NULL, NULL)
 
     assert call(E=256) == UNSUPPORTED       # fused routing only for E in {64, 128}
     assert call(E=96) == UNSUPPORTED
@@ -195,8 +195,10 @@ def test_router_route_rejects(lib):
     assert call(off=NULL) == INVALID        # loads without offsets
     assert call(M=0) == INVALID
     assert call(x=MISALIGNED) == INVALID
+    assert call(hist=MISALIGNED) == INVALID
     assert call(T=-1) == INVALID
     assert call(T=0) == 0
+    assert call(T=0, hist=FAKE) == 0
     assert call(T=0, off=NULL, loads=NULL, idx=NULL) == 0
 
 

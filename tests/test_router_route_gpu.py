@@ -44,13 +44,16 @@ def run_fused(x_bits, W_bits, b, K, offsets):
     idx = Guarded((T, K), torch.int32, fill=-7)
     tau = Guarded((T,), torch.float32, fill=-7.0)
     loads = Guarded((M, E), torch.int32)
+    H = Guarded((E, 256), torch.int32)
     err = Guarded((1,), torch.int32)
     off = torch.from_numpy(np.ascontiguousarray(offsets, np.int64)).cuda()
     eqb.eqb_router_route(to_dev_bf16(x_bits), to_dev_bf16(W_bits), torch.from_numpy(b).cuda(), K, off,
-                         z=Z.view, topk_idx=idx.view, tau=tau.view, loads=loads.view, err_flag=err.view)
+                         z=Z.view, topk_idx=idx.view, tau=tau.view, loads=loads.view, hist_hi=H.view,
+                         err_flag=err.view)
     torch.cuda.synchronize()
-    for g in (Z, idx, tau, loads, err):
+    for g in (Z, idx, tau, loads, H, err):
         assert g.intact(), "write outside an output buffer"
+    run_fused.last_hist = H.view.cpu().numpy()
     return (Z.view.view(torch.int16).cpu().numpy().view(np.uint16), idx.view.cpu().numpy(),
             tau.view.cpu().numpy(), loads.view.cpu().numpy(), int(err.view.item()))
 
@@ -71,6 +74,8 @@ def test_router_route_matches_oracle(T, d, E, K):
     np.testing.assert_array_equal(idx, i_or)
     np.testing.assert_array_equal(tau.view(np.uint32), t_or.view(np.uint32))
     np.testing.assert_array_equal(loads, l_or)
+    # the coarse histogram counted in the epilogue (Algorithm 1 step 1)
+    np.testing.assert_array_equal(run_fused.last_hist, oracle.hist_hi(z_or, t_or))
 
 
 def two_calls(x, W, b, K, off, M):
@@ -80,8 +85,9 @@ def two_calls(x, W, b, K, off, M):
     idx = torch.empty((T, K), dtype=torch.int32, device="cuda")
     tau = torch.empty(T, dtype=torch.float32, device="cuda")
     loads = torch.zeros((M, E), dtype=torch.int32, device="cuda")
-    eqb.eqb_route_topk(z, b, K, off, topk_idx=idx, tau=tau, loads=loads)
-    return z, idx, tau, loads
+    H = torch.zeros((E, 256), dtype=torch.int32, device="cuda")
+    eqb.eqb_route_topk(z, b, K, off, topk_idx=idx, tau=tau, loads=loads, hist_hi=H)
+    return z, idx, tau, loads, H
 
 
 def fused(x, W, b, K, off, M):
@@ -89,9 +95,10 @@ def fused(x, W, b, K, off, M):
     E = W.shape[0]
     idx = torch.empty((T, K), dtype=torch.int32, device="cuda")
     loads = torch.zeros((M, E), dtype=torch.int32, device="cuda")
+    H = torch.zeros((E, 256), dtype=torch.int32, device="cuda")
     err = torch.zeros(1, dtype=torch.int32, device="cuda")
-    z, idx, tau = eqb.eqb_router_route(x, W, b, K, off, topk_idx=idx, loads=loads, err_flag=err)
-    return z, idx, tau, loads, err
+    z, idx, tau = eqb.eqb_router_route(x, W, b, K, off, topk_idx=idx, loads=loads, hist_hi=H, err_flag=err)
+    return z, idx, tau, loads, err, H
 
 
 @pytest.mark.parametrize("T,d,E,K", [(5000, 4096, 128, 8), (3001, 1024, 64, 8), (777, 512, 128, 2)])
@@ -108,6 +115,7 @@ def test_router_route_equals_two_calls(T, d, E, K):
     assert torch.equal(a[1], f[1])
     assert torch.equal(a[2].view(torch.int32), f[2].view(torch.int32))
     assert torch.equal(a[3], f[3])
+    assert torch.equal(a[4], f[5])
 
 
 def test_router_route_full_size_equals_two_calls():
@@ -126,7 +134,29 @@ def test_router_route_full_size_equals_two_calls():
     assert torch.equal(a[1], f[1])
     assert torch.equal(a[2].view(torch.int32), f[2].view(torch.int32))
     assert torch.equal(a[3], f[3])
+    assert torch.equal(a[4], f[5])
     assert int(f[3].sum()) == sh.T * sh.K
+    assert torch.all(f[5].sum(1) == sh.T)
+
+
+@pytest.mark.slow
+def test_router_route_coarse_pass_beyond_the_epilogue_limit():
+    """T = 10,000,000 with d = 64: more than 65,535 tokens for some block, so
+    the coarse histogram comes from the coarse pass over z after the
+    projection; it equals the separate calls' (and so does everything
+    else)."""
+    T, d, E, K, M = 10_000_000, 64, 128, 8, 5
+    x, W = make_router_inputs(T=T, d_model=d, device="cuda", E=E)
+    b = torch.zeros(E, dtype=torch.float32, device="cuda")
+    off = torch.from_numpy(ragged_offsets(T, M, seed=9)).cuda()
+    a = two_calls(x, W, b, K, off, M)
+    f = fused(x, W, b, K, off, M)
+    torch.cuda.synchronize()
+    assert f[4].item() == 0
+    assert torch.equal(a[1], f[1])
+    assert torch.equal(a[3], f[3])
+    assert torch.equal(a[4], f[5])
+    assert torch.all(f[5].sum(1) == T)
 
 
 def test_router_route_nonfinite_bias_flagged():
