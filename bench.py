@@ -637,47 +637,12 @@ def main():
     if err:
         raise RuntimeError(f"device flagged {step.eqb.STATUS.get(err, err)}")
 
-    t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    # Inputs of the small configurations fit in L2 (129 MB): each of their
-    # steps is timed on its own, after a write of a buffer larger than L2
-    # that sits outside the timed region.
-    flush = None
-    if args.workload in ("tiny", "tie", "mid"):
-        flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
-        step_evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                    for _ in range(args.steps)]
-    clocks = ClockSampler(local)
-    barrier()
-    clocks.start()
-    time.sleep(0.3)  # let the sampler start before the timed region
-    if flush is None:
-        t_start.record(stream)
-        for s_ in range(args.steps):
-            do_step()
-        t_end.record(stream)
-    else:
-        for s_ in range(args.steps):
-            flush.fill_(s_ & 0xff)
-            step_evs[s_][0].record(stream)
-            do_step()
-            step_evs[s_][1].record(stream)
-    barrier()
-    clk = clocks.stop()
-    if flush is None:
-        ms = t_start.elapsed_time(t_end)
-    else:
-        ms = sum(a_.elapsed_time(b_) for a_, b_ in step_evs)
-        del flush
-    if world > 1:
-        tt = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
-        ms = tt.item()
-    ms_per_step = ms / args.steps
-    value = world * T / (ms_per_step / 1e3)
-
-    # The same step captured once as a CUDA graph and replayed (launch
-    # overheads removed); reported beside the stream timing, not instead.
-    graph = None
+    # On one GPU the one-call step is also captured once as a CUDA graph,
+    # whose replay is timed by the same loop after the headline (without the
+    # host's per-launch overhead; for the steps timed one at a time a graph
+    # launch costs more than it saves).  Several GPUs run the per-pass calls
+    # with the all-reduces between them.
+    cg, graph_err = None, None
     if one_call:
         try:
             cg = torch.cuda.CUDAGraph()
@@ -686,19 +651,60 @@ def main():
             torch.cuda.synchronize()
             with torch.cuda.graph(cg, stream=gs, capture_error_mode="relaxed"):
                 step.run_step(gs)
-            rs = torch.cuda.current_stream()  # replay() launches on the current stream
-            cg.replay()
             torch.cuda.synchronize()
-            ga, gb = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            ga.record(rs)
+            cg.replay()  # replay() launches on the current stream
+            torch.cuda.synchronize()
+        except Exception as exc:  # capture not possible: say why, time the stream loop
+            cg, graph_err = None, f"{type(exc).__name__}: {exc}"[:200]
+
+    # Inputs of the small configurations fit in L2 (129 MB): each of their
+    # steps is timed on its own, after a write of a buffer larger than L2
+    # that sits outside the timed region.
+    flush = None
+    if args.workload in ("tiny", "tie", "mid"):
+        flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
+
+    def timed_loop(fn):
+        """Milliseconds of args.steps steps of fn, by CUDA events on the stream."""
+        if flush is None:
+            t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            t_start.record(stream)
             for _ in range(args.steps):
-                cg.replay()
-            gb.record(rs)
-            torch.cuda.synchronize()
-            graph = {"ms_per_step": ga.elapsed_time(gb) / args.steps, "steps": args.steps}
-            del cg
-        except Exception as exc:  # capture not possible: say why instead of a number
-            graph = {"error": f"{type(exc).__name__}: {exc}"[:200]}
+                fn()
+            t_end.record(stream)
+            barrier()
+            return t_start.elapsed_time(t_end)
+        evs_ = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                for _ in range(args.steps)]
+        for s_ in range(args.steps):
+            flush.fill_(s_ & 0xff)
+            evs_[s_][0].record(stream)
+            fn()
+            evs_[s_][1].record(stream)
+        barrier()
+        return sum(a_.elapsed_time(b_) for a_, b_ in evs_)
+
+    clocks = ClockSampler(local)
+    barrier()
+    clocks.start()
+    time.sleep(0.3)  # let the sampler start before the timed region
+    ms = timed_loop(do_step)
+    clk = clocks.stop()
+    graph_ms = timed_loop(cg.replay) / args.steps if cg is not None else None
+    del flush
+    err = step.ws.err.item()
+    if err:
+        raise RuntimeError(f"device flagged {step.eqb.STATUS.get(err, err)}")
+    if cg is not None:
+        del cg
+    if world > 1:
+        tt = torch.tensor([ms], device=dev)
+        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        ms = tt.item()
+    ms_per_step = ms / args.steps
+    value = world * T / (ms_per_step / 1e3)
+    graph = ({"ms_per_step": graph_ms, "steps": args.steps} if graph_ms is not None else
+             {"error": graph_err} if graph_err else None)
 
     # Per-kernel durations: the same work issued kernel by kernel on one
     # stream, each launch bracketed by CUDA events, in its own timed loop.
