@@ -115,6 +115,34 @@ def summarize_clock_lines(lines):
             "sm_max_mhz": max(mx) if mx else None, "reasons": reasons, "samples": len(rows)}
 
 
+def time_steps(stream, steps, fn, flush=None, sync=torch.cuda.synchronize):
+    """Milliseconds of `steps` calls of fn, by CUDA events on `stream`: one
+    event pair around the loop, or, with `flush` (a buffer larger than L2),
+    one pair around each step, the buffer rewritten before each outside the
+    timed region."""
+    if flush is None:
+        a_, b_ = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        a_.record(stream)
+        for _ in range(steps):
+            fn()
+        b_.record(stream)
+        sync()
+        return a_.elapsed_time(b_)
+    evs = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)) for _ in range(steps)]
+    for s_ in range(steps):
+        flush.fill_(s_ & 0xff)
+        evs[s_][0].record(stream)
+        fn()
+        evs[s_][1].record(stream)
+    sync()
+    return sum(a_.elapsed_time(b_) for a_, b_ in evs)
+
+
+# Workloads whose inputs fit in L2 (129 MB): each step is timed on its own
+# after a write of a buffer larger than L2.
+SMALL_WORKLOADS = ("tiny", "tie", "mid")
+
+
 class Step:
     """Device buffers and the launch sequence of one routing-balance step.
 
@@ -583,6 +611,47 @@ def extras(step, stream, peak):
     return out
 
 
+# Steps timed for each of the other workloads in the default run.
+OTHER_STEPS = {"tiny": 100, "tie": 50, "mid": 20, "router": 10, "paper": 10, "wide": 20}
+
+
+def other_workloads(dev, stream, peak, local, skip):
+    """The other workloads at their full sizes, each timed the way the
+    headline is (the one-call step, three warm-up steps, CUDA events; the
+    small ones a step at a time after an L2-evicting write), with its own
+    clock record, so that one run of the benchmark measures all of them."""
+    out = {}
+    for w, n in OTHER_STEPS.items():
+        if w == skip:
+            continue
+        sh = SHAPES[w]
+        st = Step(w, sh.T, dev)
+        st.r_global = st.eqb.eqb_target_rank(sh.T, st.E, st.K)
+
+        def fn():
+            st.run_step(stream)
+
+        for _ in range(3):
+            fn()
+        torch.cuda.synchronize()
+        flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev) if w in SMALL_WORKLOADS else None
+        clocks = ClockSampler(local)
+        clocks.start()
+        time.sleep(0.3)
+        ms = time_steps(stream, n, fn, flush) / n
+        clk = clocks.stop()
+        err = st.ws.err.item()
+        gbs = st.algorithmic_bytes()["path"] / (ms * 1e-3) / 1e9
+        out[w] = {"ms_per_step": ms, "tokens_per_s": sh.T / (ms * 1e-3), "path_GB/s": round(gbs, 1),
+                  "path_frac": round(gbs / peak, 4), "steps": n, "warmup": 3,
+                  "T": sh.T, "E": st.E, "K": st.K, "M": st.M,
+                  "l2": "per-step eviction" if flush is not None else "inputs larger than L2", "clocks": clk,
+                  **({"device_error": st.eqb.STATUS.get(err, err)} if err else {})}
+        del st, flush
+        torch.cuda.empty_cache()
+    return out
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -657,40 +726,14 @@ def main():
         except Exception as exc:  # capture not possible: say why, time the stream loop
             cg, graph_err = None, f"{type(exc).__name__}: {exc}"[:200]
 
-    # Inputs of the small configurations fit in L2 (129 MB): each of their
-    # steps is timed on its own, after a write of a buffer larger than L2
-    # that sits outside the timed region.
-    flush = None
-    if args.workload in ("tiny", "tie", "mid"):
-        flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev)
-
-    def timed_loop(fn):
-        """Milliseconds of args.steps steps of fn, by CUDA events on the stream."""
-        if flush is None:
-            t_start, t_end = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-            t_start.record(stream)
-            for _ in range(args.steps):
-                fn()
-            t_end.record(stream)
-            barrier()
-            return t_start.elapsed_time(t_end)
-        evs_ = [(torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
-                for _ in range(args.steps)]
-        for s_ in range(args.steps):
-            flush.fill_(s_ & 0xff)
-            evs_[s_][0].record(stream)
-            fn()
-            evs_[s_][1].record(stream)
-        barrier()
-        return sum(a_.elapsed_time(b_) for a_, b_ in evs_)
-
+    flush = torch.empty(512 << 20, dtype=torch.uint8, device=dev) if args.workload in SMALL_WORKLOADS else None
     clocks = ClockSampler(local)
     barrier()
     clocks.start()
     time.sleep(0.3)  # let the sampler start before the timed region
-    ms = timed_loop(do_step)
+    ms = time_steps(stream, args.steps, do_step, flush, barrier)
     clk = clocks.stop()
-    graph_ms = timed_loop(cg.replay) / args.steps if cg is not None else None
+    graph_ms = time_steps(stream, args.steps, cg.replay, flush, barrier) / args.steps if cg is not None else None
     del flush
     err = step.ws.err.item()
     if err:
@@ -792,6 +835,9 @@ def main():
     ext = None
     if rank == 0 and world == 1 and not args.no_extras and args.workload != "router":
         ext = extras(step, stream, peak)
+    others = None
+    if rank == 0 and world == 1 and not args.no_extras and args.tokens is None:
+        others = other_workloads(dev, stream, peak, local, args.workload)
 
     if rank == 0:
         line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world,
@@ -804,7 +850,7 @@ def main():
                                         f"{args.workload}: T={T} E={E} K={K} M={M} per GPU, bf16 logits"),
                            "T": T, "E": E, "K": K, "M": M, "eta": ETA, "c": C_NORM,
                            "l2": ("each step timed alone after a 512 MiB write that evicts L2 (outside the "
-                                  "timed region)" if args.workload in ("tiny", "tie", "mid") else
+                                  "timed region)" if args.workload in SMALL_WORKLOADS else
                                   "inputs larger than L2 (at least 1 GiB each); no flush"),
                            "parallelism": f"dp{world}"},
                 "gpu_launches": step.launches_per_step() * args.steps,
@@ -815,7 +861,8 @@ def main():
                 "kernels": kernels,
                 "kernels_sequential_ms": seq_ms,
                 "clocks": clk, "e2e": e2e, "cpu_baseline": cpu_base,
-                "elements_per_s": value * E, "cuda_graph": graph, "extras": ext}
+                "elements_per_s": value * E, "cuda_graph": graph, "extras": ext,
+                "other_workloads": others}
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()
