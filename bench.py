@@ -764,7 +764,8 @@ def main():
     seq_ms = sum(per_kernel.values())
     alg = step.algorithmic_bytes()
     peak, peak_kind = measured_peaks()
-    dom = max(per_kernel, key=per_kernel.get)
+    # the roofline's kernel: the slowest of those with algorithmic bytes
+    dom = max((k for k in per_kernel if k in alg), key=per_kernel.get)
     dom_bytes = alg.get(dom)
     traffic = dram_traffic(args.traffic_file, dom, T, E)
     achieved = dom_bytes / (per_kernel[dom] * 1e-3) / 1e9

@@ -140,6 +140,42 @@ def test_router_route_full_size_equals_two_calls():
 
 
 @pytest.mark.slow
+def test_router_route_epilogue_counters_at_their_limit():
+    """The largest T whose coarse histogram is still counted in the
+    epilogue: every block takes 511 tiles (65,408 tokens), so each 16-bit
+    window counter climbs to 65,408 when all tokens agree.  Constant
+    integer rows make every token's logits, top-K, cutoff and margins the
+    same (b = 0), so H = T x the histogram of one row (Algorithm 1 step 1)
+    and each microbatch's loads are its size on the row's top-K."""
+    sms = torch.cuda.get_device_properties(0).multi_processor_count
+    T, d, E, K = 511 * sms * 128, 64, 128, 8
+    xr, W, _ = integer_inputs(1, d, E, seed=21)
+    b = np.zeros(E, np.float32)
+    offsets = ragged_offsets(T, 3, seed=4)
+    x = to_dev_bf16(xr).expand(T, d).contiguous()
+    idx = torch.empty((T, K), dtype=torch.int32, device="cuda")
+    loads = torch.zeros((3, E), dtype=torch.int32, device="cuda")
+    H = torch.zeros((E, 256), dtype=torch.int32, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    z, idx, tau = eqb.eqb_router_route(x, to_dev_bf16(W), torch.from_numpy(b).cuda(), K,
+                                       torch.from_numpy(offsets).cuda(), topk_idx=idx, loads=loads,
+                                       hist_hi=H, err_flag=err)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    del x
+    zr, _ = oracle.router_logits(xr, W, np.arange(1))
+    z_row = brute.bf16_bits_from_f32(zr.astype(np.float32))
+    i_row, t_row, _ = oracle.route(z_row, b, K, np.array([0, 1], np.int64))
+    assert torch.equal(z[0].view(torch.int16).cpu(), torch.from_numpy(z_row[0].view(np.int16)))
+    assert bool((idx == torch.from_numpy(i_row[0]).cuda()).all())
+    assert bool((tau.view(torch.int32) == int(t_row.view(np.int32)[0])).all())
+    np.testing.assert_array_equal(H.cpu().numpy(), T * oracle.hist_hi(z_row, t_row).astype(np.int64))
+    want = np.zeros((3, E), np.int64)
+    want[:, i_row[0]] = np.diff(offsets)[:, None]
+    np.testing.assert_array_equal(loads.cpu().numpy(), want)
+
+
+@pytest.mark.slow
 def test_router_route_coarse_pass_beyond_the_epilogue_limit():
     """T = 10,000,000 with d = 64: more than 65,535 tokens for some block, so
     the coarse histogram comes from the coarse pass over z after the
