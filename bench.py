@@ -50,6 +50,19 @@ def dist_env():
     return ws, rank, local
 
 
+def allreduce_(t, op=None):
+    """t summed (or reduced by op) over the ranks, in place.  NCCL reduces
+    device tensors; another backend (gloo) goes through host memory."""
+    import torch.distributed as dist
+    op = dist.ReduceOp.SUM if op is None else op
+    if dist.get_backend() == "nccl":
+        dist.all_reduce(t, op=op)
+    else:
+        h = t.cpu()
+        dist.all_reduce(h, op=op)
+        t.copy_(h)
+
+
 def measured_peaks():
     p = os.path.join(ROOT, "MEASURED_PEAKS.json")
     if os.path.exists(p):
@@ -253,7 +266,7 @@ class Step:
             rec(0, lambda: eqb.eqb_router_route(self.x, self.W, self.b, self.K, self.off, z, self.idx,
                                                 self.tau, self.loads, ws.err, stream, hist_hi=ws.hist_hi))
             if world > 1:
-                torch.distributed.all_reduce(ws.hist_hi)
+                allreduce_(ws.hist_hi)
             k = 1
             if self.fused:
                 rec(1, lambda: eqb.lei_coefficients(self.loads, self.off, self.K, ETA, C_NORM, self.coef, stream))
@@ -265,7 +278,7 @@ class Step:
             else:
                 rec(k + 1, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
             if world > 1:
-                torch.distributed.all_reduce(ws.hist_lo)
+                allreduce_(ws.hist_lo)
             rec(k + 2, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err, stream))
             rec(k + 3, lambda: eqb.eqb_bias_update(ws.q_hat, self.b_next, stream))
             if not self.fused:
@@ -282,7 +295,7 @@ class Step:
         else:
             rec(1, lambda: eqb.eqb_margin_hist_pass1(z, self.tau, ws.hist_hi, ws.err, stream))
         if world > 1:
-            torch.distributed.all_reduce(ws.hist_hi)
+            allreduce_(ws.hist_hi)
         k = 3 if self.fused else 2
         rec(k, lambda: eqb.eqb_select_quantile(ws.hist_hi, 1, r, ws.u, ws.rho, None, ws.err, stream))
         if self.fused:
@@ -291,7 +304,7 @@ class Step:
         else:
             rec(3, lambda: eqb.eqb_margin_hist_pass2(z, self.tau, ws.u, ws.hist_lo, stream))
         if world > 1:
-            torch.distributed.all_reduce(ws.hist_lo)
+            allreduce_(ws.hist_lo)
         k += 2
         rec(k, lambda: eqb.eqb_select_quantile(ws.hist_lo, 2, r, ws.u, ws.rho, ws.q_hat, ws.err,
                                                     stream))
@@ -675,8 +688,14 @@ def main():
         return run_reference(args)
 
     world, rank, local = dist_env()
+    # EQB_BENCH_BACKEND and EQB_BENCH_DEVICE run the multi-rank path with
+    # another process-group backend or on a chosen device: two ranks on one
+    # GPU through gloo exchange their histograms through host memory, which
+    # checks that the path runs and agrees across ranks (not a scaling
+    # measurement).
     if world > 1:
-        torch.distributed.init_process_group("nccl")
+        torch.distributed.init_process_group(os.environ.get("EQB_BENCH_BACKEND", "nccl"))
+    local = int(os.environ.get("EQB_BENCH_DEVICE", local))
     torch.cuda.set_device(local)
     dev = torch.device("cuda", local)
     sh = SHAPES[args.workload]
@@ -742,10 +761,18 @@ def main():
         del cg
     if world > 1:
         tt = torch.tensor([ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        allreduce_(tt, torch.distributed.ReduceOp.MAX)
         ms = tt.item()
     ms_per_step = ms / args.steps
     value = world * T / (ms_per_step / 1e3)
+    # Every rank forms the next bias from the same summed histograms, so the
+    # ranks must agree bit for bit.
+    ranks_agree = None
+    if world > 1:
+        mine = step.b_next.cpu()
+        every = [torch.empty_like(mine) for _ in range(world)]
+        torch.distributed.all_gather_object(every, mine)
+        ranks_agree = all(torch.equal(mine.view(torch.int32), o.view(torch.int32)) for o in every)
     graph = ({"ms_per_step": graph_ms, "steps": args.steps} if graph_ms is not None else
              {"error": graph_err} if graph_err else None)
 
@@ -812,7 +839,7 @@ def main():
         barrier()
         e_ms = a.elapsed_time(bq) / args.e2e_steps
         tt = torch.tensor([e_ms], device=dev)
-        torch.distributed.all_reduce(tt, op=torch.distributed.ReduceOp.MAX)
+        allreduce_(tt, torch.distributed.ReduceOp.MAX)
         e_ms = tt.item()
         e2e = {"value": world * T / (e_ms / 1e3), "unit": "tokens/s", "h2d_bytes_per_step": h2d,
                "d2h_bytes_per_step": d2h, "ms_per_step": e_ms, "schedule": "serial on one stream"}
@@ -863,7 +890,8 @@ def main():
                 "kernels_sequential_ms": seq_ms,
                 "clocks": clk, "e2e": e2e, "cpu_baseline": cpu_base,
                 "elements_per_s": value * E, "cuda_graph": graph, "extras": ext,
-                "other_workloads": others}
+                "other_workloads": others,
+                **({"ranks_agree": ranks_agree} if world > 1 else {})}
         print(json.dumps(line), flush=True)
     if world > 1:
         torch.distributed.destroy_process_group()

@@ -6,7 +6,8 @@ counts inside the selected bins (step 5).  These tests shard a batch across
 two processes the way bench.py does under torchrun (contiguous token ranges,
 global target rank), all-reduce the per-rank counts with torch.distributed,
 and check that both ranks recover the single-process quantile and bias.
-The per-rank counts come from the oracle (no GPU here)."""
+The sums go through bench.py's own all-reduce helper.  The per-rank counts
+come from the oracle (no GPU here)."""
 import os
 import socket
 import sys
@@ -39,6 +40,7 @@ def _worker(rank, world, port, T, E, K, seed, out_q):
     try:
         import brute
         import oracle
+        from bench import allreduce_
         rng = np.random.default_rng(seed)
         z = brute.bf16_bits_from_f32(rng.standard_normal((T, E)).astype(np.float32))
         b = (rng.standard_normal(E) * 0.2).astype(np.float32)
@@ -47,10 +49,10 @@ def _worker(rank, world, port, T, E, K, seed, out_q):
         _, tau, _ = oracle.route(zl, b, K)
         r = oracle.target_rank(T, E, K)          # global rank, as in Algorithm 1
         H = torch.from_numpy(oracle.hist_hi(zl, tau))
-        dist.all_reduce(H)                        # step 2
+        allreduce_(H)                             # step 2
         u, rho = oracle.select_hi(H.numpy(), r)   # step 3
         L = torch.from_numpy(oracle.hist_lo(zl, tau, u))
-        dist.all_reduce(L)                        # step 5
+        allreduce_(L)                             # step 5
         q = oracle.select_lo(L.numpy(), u, rho)   # steps 5-6
         out_q.put((rank, q.tolist(), oracle.bias_update(q).view(np.uint32).tolist()))
     finally:
