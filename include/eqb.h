@@ -366,8 +366,8 @@ eqb_status eqb_maxvio(const int32_t *loads, const int64_t *mb_offsets, int32_t M
  *               hist_hi [E,256] += (nullable): the coarse histogram, counted
  *               in the same kernel from the rows it just stored (read back
  *               from L2) when no block of the kernel routes more than 65,535
- *               tokens (T <= 65,535 x the SM count, rounded down to 128-row
- *               tiles), else by the coarse pass over z after it
+ *               tokens (T <= 65,408 x the SM count: 511 tiles of 128 rows per
+ *               block), else by the coarse pass over z after it
  * Results equal those of the calls made one after the other on the same
  * inputs, bit for bit.  err_flag: EQB_ERR_NONFINITE as in eqb_route_topk,
  * EQB_ERR_CUDA as in eqb_router_logits.
