@@ -95,9 +95,10 @@ __device__ __forceinline__ void route_row(const uint8_t* rowp, const float* bs, 
   for (int c = NH; c < NP; ++c) cm[c] = 0xff80ff80u;
 #pragma unroll
   for (int c = 0; c < NH; ++c) {
-    // At E > 256 the unrolled loads would not fit in registers if all were
-    // hoisted: let at most eight pairs of chunks be in flight.
-    if (NH > 16 && c > 0 && (c & 7) == 0) asm volatile("" ::: "memory");
+    // From E = 256 on the unrolled loads do not fit in registers if all are
+    // hoisted (at E = 256 the 168 registers of a 12-warp block spilled):
+    // let at most eight pairs of chunks be in flight.
+    if (NH > 8 && c > 0 && (c & 7) == 0) asm volatile("" ::: "memory");
     const uint32_t qa = chunk_max(lds128(rowp + 16 * c), bdn4[c]);
     const uint32_t qb = chunk_max(lds128(rowp + 16 * (c + NH)), bdn4[c + NH]);
     cm[c] = hmax2_nan_bf16(prmt(qa, qb, 0x5410u), prmt(qa, qb, 0x7632u));
