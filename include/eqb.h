@@ -53,7 +53,7 @@ typedef uint16_t eqb_bf16; /* raw bf16 bit pattern */
 typedef enum eqb_status {
   EQB_OK = 0,
   EQB_ERR_INVALID_ARG = 1, /* host-side validation failed; nothing launched */
-  EQB_ERR_UNSUPPORTED = 2, /* valid by the paper, outside this build's sizes */
+  EQB_ERR_UNSUPPORTED = 2, /* valid by the paper, outside the sizes the library supports */
   EQB_ERR_CUDA = 3,        /* a CUDA launch or runtime call failed */
   EQB_ERR_NONFINITE = 4,   /* device flag: non-finite z, b or score, or a
                               margin of magnitude >= 2^127 */

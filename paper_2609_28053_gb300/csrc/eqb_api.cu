@@ -43,7 +43,7 @@ namespace {
 
 inline bool aligned(const void* p, uintptr_t a) { return (reinterpret_cast<uintptr_t>(p) % a) == 0; }
 
-// Sizes this build supports (the paper allows 1 <= K < E).
+// Sizes the library supports (the paper allows 1 <= K < E).
 inline eqb_status check_shape(int64_t T, int32_t E, int32_t K, bool need_k) {
   if (T < 0 || E < 2) return EQB_ERR_INVALID_ARG;
   if (need_k && (K < 1 || K >= E)) return EQB_ERR_INVALID_ARG;
