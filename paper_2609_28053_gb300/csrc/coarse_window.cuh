@@ -66,8 +66,8 @@ __device__ __forceinline__ void coarse_window_outside_body(uint32_t y, uint32_t 
 // busy (the router projection's x stream): there an instruction fetch that
 // misses the cache costs far more than the call, so the counting loop is kept
 // small.
-static __device__ __noinline__ void coarse_window_outside(uint32_t y, uint32_t k, uint32_t crow, uint32_t zword, int e0,
-                                                   int32_t* hist, int32_t* err) {
+static __device__ __noinline__ void coarse_window_outside(uint32_t y, uint32_t k, uint32_t crow, uint32_t zword,
+                                                          int e0, int32_t* hist, int32_t* err) {
   coarse_window_outside_body(y, k, crow, zword, e0, hist, err);
 }
 
