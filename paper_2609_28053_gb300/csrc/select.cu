@@ -19,13 +19,17 @@ namespace eqb {
 
 namespace {
 
+constexpr int kSelectBiasMaxE = 1024;  // experts of one select_bias_kernel block
+
 // One warp selects for expert e from its 256 counts, lane j holding bins
 // 8j..8j+7 (cnt): pass 1 writes u[e] and rho[e] for the rank `target`, pass 2
-// writes q_hat[e] from u[e] and the rank target = rho[e].  Flags a count in
+// writes q_hat[e] (and *qs, when given) from u_e = u[e] and the rank target =
+// rho[e], both read by the caller beside the counts.  Flags a count in
 // high-byte bin 0x00 or 0xff (pass 1) and an unreachable rank.
 __device__ __forceinline__ void warp_select(const int64_t (&cnt)[8], int e, int pass, int64_t target,
-                                            uint8_t* __restrict__ u, int32_t* __restrict__ rho,
-                                            uint16_t* __restrict__ q_hat, int32_t* err, int lane) {
+                                            uint32_t u_e, uint8_t* __restrict__ u, int32_t* __restrict__ rho,
+                                            uint16_t* __restrict__ q_hat, int32_t* err, int lane,
+                                            uint16_t* qs = nullptr) {
   int64_t local = 0;
 #pragma unroll
   for (int j = 0; j < 8; ++j) local += cnt[j];
@@ -44,7 +48,10 @@ __device__ __forceinline__ void warp_select(const int64_t (&cnt)[8], int e, int 
     if (lane == 0) {
       raise_flag(err, kErrRank);
       if (first) { u[e] = 255; rho[e] = 0; }
-      else q_hat[e] = 0x7fc0;  // NaN marks an unreachable rank
+      else {
+        q_hat[e] = 0x7fc0;  // NaN marks an unreachable rank
+        if (qs) *qs = 0x7fc0;
+      }
     }
     return;
   }
@@ -58,9 +65,10 @@ __device__ __forceinline__ void warp_select(const int64_t (&cnt)[8], int e, int 
           u[e] = static_cast<uint8_t>(bin);
           rho[e] = static_cast<int32_t>(target - below);
         } else {
-          uint32_t q = kappa16_inv((static_cast<uint32_t>(u[e]) << 8) | static_cast<uint32_t>(bin));
+          uint32_t q = kappa16_inv((u_e << 8) | static_cast<uint32_t>(bin));
           if (q == 0x8000u) q = 0u;
           q_hat[e] = static_cast<uint16_t>(q);
+          if (qs) *qs = static_cast<uint16_t>(q);
         }
         break;
       }
@@ -99,7 +107,9 @@ __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__
   int64_t cnt[8];
 #pragma unroll
   for (int j = 0; j < 8; ++j) cnt[j] = h[j];
-  warp_select(cnt, e, pass, pass != 2 ? r : (int64_t)rho[e], u, rho, q_hat, err, lane);
+  const int64_t target = pass != 2 ? r : (int64_t)rho[e];
+  const uint32_t u_e = pass == 2 ? u[e] : 0u;
+  warp_select(cnt, e, pass, target, u_e, u, rho, q_hat, err, lane);
 }
 
 // Exponent range of a non-zero bf16 pattern: [ulp exponent, leading-bit exponent].
@@ -117,17 +127,20 @@ __device__ __forceinline__ void bf16_exp_range(uint32_t x, int& lo, int& hi) {
 // tree reduction reproduces the sequential sum bit for bit.  Otherwise one
 // thread sums in ascending order.
 // The block computes b_next from q_hat (the threads of the block share the
-// final subtraction; warp 0 forms the mean).
+// final subtraction; warp 0 forms the mean).  SHARED_Q: q_hat is the block's
+// shared-memory copy; otherwise the global array, read through L2 (it may
+// have been written earlier in the same kernel).
+template <bool SHARED_Q>
 __device__ __forceinline__ void block_bias_update(const uint16_t* q_hat, int E, float* __restrict__ b_next) {
   __shared__ double mean;
-  // q_hat may have been written earlier in the same kernel: read it through L2
+  auto q_at = [&](int e) -> uint32_t { return SHARED_Q ? q_hat[e] : __ldcg(q_hat + e); };
 
   if (threadIdx.x < 32) {
     const int lane = threadIdx.x;
     double part = 0.0;
     int lo = 1 << 20, hi = -(1 << 20);
     for (int e = lane; e < E; e += 32) {
-      const uint32_t x = __ldcg(q_hat + e);
+      const uint32_t x = q_at(e);
       if ((x & 0x7fffu) != 0u) {
         int l, h;
         bf16_exp_range(x, l, h);
@@ -150,51 +163,59 @@ __device__ __forceinline__ void block_bias_update(const uint16_t* q_hat, int E, 
     } else {
       sum = 0.0;
       if (lane == 0)
-        for (int e = 0; e < E; ++e) sum = __dadd_rn(sum, (double)bf16_bits_to_f32(__ldcg(q_hat + e)));
+        for (int e = 0; e < E; ++e) sum = __dadd_rn(sum, (double)bf16_bits_to_f32(q_at(e)));
     }
     if (lane == 0) mean = __ddiv_rn(sum, (double)E);
   }
   __syncthreads();
   for (int e = threadIdx.x; e < E; e += blockDim.x)
-    b_next[e] = __double2float_rn(__dsub_rn((double)bf16_bits_to_f32(__ldcg(q_hat + e)), mean));
+    b_next[e] = __double2float_rn(__dsub_rn((double)bf16_bits_to_f32(q_at(e)), mean));
 }
 
 
 __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, float* __restrict__ b_next) {
   griddep_wait();
-  block_bias_update(q_hat, E, b_next);
+  block_bias_update<false>(q_hat, E, b_next);
 }
 
 // Algorithm 1 steps 5-6 and Eq. (2) in one block: the pass-2 selection of
-// every expert (each warp loads the counts of 4 experts before it scans
-// them), then the bias update.  Same results as select_kernel (pass 2)
-// followed by bias_update_kernel.
+// every expert (each warp loads the counts, rho and u of 4 experts before it
+// scans them, so a batch costs one L2 round trip), then the bias update from
+// the block's shared copy of q_hat.  Same results as select_kernel (pass 2)
+// followed by bias_update_kernel.  E <= kSelectBiasMaxE.
 __global__ void __launch_bounds__(1024) select_bias_kernel(const int32_t* __restrict__ hist, int E,
                                                            const uint8_t* __restrict__ u,
                                                            int32_t* __restrict__ rho,
                                                            uint16_t* __restrict__ q_hat, int32_t* err,
                                                            float* __restrict__ b_next) {
   constexpr int B = 4;
+  __shared__ uint16_t qs[kSelectBiasMaxE];
   griddep_wait();
   const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
   for (int e0 = wid; e0 < E; e0 += nw * B) {
     int4 ca[B], cb[B];
+    int32_t rk[B];
+    uint32_t uk = 0u;  // u of the batch, one byte per expert
 #pragma unroll
     for (int k = 0; k < B; ++k) {
-      const int e = e0 + k * nw;
-      const int32_t* h = hist + (int64_t)min(e, E - 1) * 256 + lane * 8;
+      const int e = min(e0 + k * nw, E - 1);
+      const int32_t* h = hist + (int64_t)e * 256 + lane * 8;
       ca[k] = __ldg(reinterpret_cast<const int4*>(h));
       cb[k] = __ldg(reinterpret_cast<const int4*>(h + 4));
+      rk[k] = __ldcg(rho + e);
+      uk |= static_cast<uint32_t>(__ldcg(u + e)) << (8 * k);
     }
 #pragma unroll
     for (int k = 0; k < B; ++k) {
       const int e = e0 + k * nw;
       const int64_t cnt[8] = {ca[k].x, ca[k].y, ca[k].z, ca[k].w, cb[k].x, cb[k].y, cb[k].z, cb[k].w};
-      if (e < E) warp_select(cnt, e, 2, (int64_t)rho[e], const_cast<uint8_t*>(u), rho, q_hat, err, lane);
+      if (e < E)
+        warp_select(cnt, e, 2, (int64_t)rk[k], (uk >> (8 * k)) & 0xffu, const_cast<uint8_t*>(u), rho, q_hat, err,
+                    lane, qs + e);
     }
   }
   __syncthreads();  // every q_hat is written
-  block_bias_update(q_hat, E, b_next);
+  block_bias_update<true>(qs, E, b_next);
 }
 
 }  // namespace
@@ -221,6 +242,7 @@ int launch_select_sharded(const int32_t* hist, int E, int pass, const int64_t* s
 
 int launch_select_bias(const int32_t* hist, int E, const uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err,
                        float* b_next, cudaStream_t s) {
+  if (E > kSelectBiasMaxE) return kErrUnsupported;
   return launch_dependent(select_bias_kernel, dim3(1), dim3(1024), 0, s, hist, E, u, rho, q_hat, err, b_next) ==
                  cudaSuccess
              ? kOk
