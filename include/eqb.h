@@ -164,8 +164,9 @@ eqb_status eqb_bias_update(const eqb_bf16 *q_hat, int32_t E, float *b_next,
  *   c > 0:  xi = max_e |rho_e| / c,  sigma = tanh(xi) / xi (1 at xi = 0);
  *   c <= 0: sigma = 1 (unnormalised LEI);
  *   grad_s[t, e] += eta * sigma * rho_e for every t in the microbatch and
- *   every expert e.  The coefficient is formed in fp64, rounded to fp32,
- *   and added in fp32.
+ *   every expert e.  rho and the product eta * sigma * rho are formed in
+ *   fp64 (sigma in fp32, within a few fp32 ulps of tanh(xi) / xi), rounded
+ *   to fp32, and added in fp32.
  *   grad_s  device fp32 [T,E], 16-byte aligned, updated in place
  *   loads   device int32 [M,E] (the local loads from eqb_route_topk) */
 eqb_status lei_inject_grad(float *grad_s, const int32_t *loads,
@@ -174,8 +175,8 @@ eqb_status lei_inject_grad(float *grad_s, const int32_t *loads,
 
 /* The Load-Error Injection coefficients (Sec. 4, Eqs. LEI and norm) as a
  * table: coef[l, e] = (float)(eta * sigma_l * rho_{l,e}), rho and sigma of
- * microbatch l as in lei_inject_grad, by the same fp64 arithmetic (so the
- * same bits as the coefficient lei_inject_grad adds).  An empty microbatch
+ * microbatch l as in lei_inject_grad, by the same arithmetic (so the same
+ * bits as the coefficient lei_inject_grad adds).  An empty microbatch
  * gets a row of zeros.
  *   loads  device int32 [M,E]                          (in)
  *   coef   device fp32 [M,E], 16-byte aligned          (out) */

@@ -57,12 +57,15 @@ __device__ void block_lei_coef(const int32_t* __restrict__ f, int64_t n, int E, 
   if (threadIdx.x == 0) {
     double rmax = red[0];
     for (int w = 1; w < kLeiThreads / 32; ++w) rmax = fmax(rmax, red[w]);
-    double sigma = 1.0;
+    // sigma = tanh(xi) / xi in fp32: its relative error (a few ulp of fp32)
+    // stays far inside the LEI tolerance, and it spares the serial fp64
+    // division and tanh of this thread
+    float sigma = 1.0f;
     if (c > 0.0f) {
-      const double xi = rmax / (double)c;
-      sigma = (xi == 0.0) ? 1.0 : tanh(xi) / xi;
+      const float xi = __fdiv_rn(static_cast<float>(rmax), c);
+      sigma = (xi == 0.0f) ? 1.0f : __fdiv_rn(tanhf(xi), xi);
     }
-    scal[1] = (double)eta * sigma;
+    scal[1] = (double)eta * (double)sigma;
   }
   __syncthreads();
 #pragma unroll
