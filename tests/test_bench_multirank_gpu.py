@@ -23,7 +23,7 @@ def _free_port():
         return s.getsockname()[1]
 
 
-@pytest.mark.parametrize("workload,tokens", [("global", 131072), ("tie", 65536)])
+@pytest.mark.parametrize("workload,tokens", [("global", 131072), ("tie", 65536), ("router", 65536)])
 def test_two_ranks_on_one_gpu_agree(cuda_ok, workload, tokens):
     env = dict(os.environ, EQB_BENCH_BACKEND="gloo", EQB_BENCH_DEVICE="0")
     cmd = [sys.executable, "-m", "torch.distributed.run", "--nnodes=1", "--nproc-per-node", "2",
