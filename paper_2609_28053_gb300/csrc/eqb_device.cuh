@@ -21,10 +21,17 @@ constexpr unsigned kFull = 0xffffffffu;
 // its block-local set-up overlap the previous kernel's drain; each kernel
 // calls griddep_wait() before it touches global memory (it returns once the
 // previous grid has completed and its writes are visible; a no-op for a grid
-// not launched as a dependent).  No kernel triggers its successor early:
-// measured on the global step, early triggers cost 60 us, while the implicit
-// trigger at completion saves 17 us against plain launches.
+// not launched as a dependent).  The implicit trigger at completion saves
+// 17 us on the global step against plain launches.  Only the short kernels
+// that precede a histogram pass (the LEI coefficient table, a selection)
+// trigger their successor early, at their start: the pass's blocks take the
+// SMs those leave idle and zero their bins meanwhile (1-3 us per step on
+// every workload).  Early triggers in every kernel cost 60 us on the global
+// step.
 __device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+// Let the next kernel in the stream launch now (it still waits, in
+// griddep_wait, for this grid to complete).
+__device__ __forceinline__ void griddep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
 
 // Launch `kern` as a programmatic dependent of the previous work in `s`.
 template <typename... KArgs, typename... Args>

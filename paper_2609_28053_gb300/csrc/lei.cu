@@ -139,6 +139,7 @@ __global__ void __launch_bounds__(kLeiThreads) lei_kernel(LeiArgs a, int64_t tok
 // One block per microbatch: row l of the [M,E] coefficient table.
 __global__ void __launch_bounds__(kLeiThreads) lei_coef_kernel(LeiArgs a, float* coef) {
   griddep_wait();
+  griddep_launch();
   const int l = blockIdx.x;
   const int64_t n = __ldg(a.off + l + 1) - __ldg(a.off + l);
   block_lei_coef(a.loads + (int64_t)l * a.E, n, a.E, a.K, a.eta, a.c, coef + (int64_t)l * a.E);

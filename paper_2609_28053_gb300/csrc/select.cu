@@ -83,6 +83,7 @@ __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__
                                                      uint16_t* __restrict__ q_hat, int32_t* err,
                                                      const int64_t* __restrict__ shard_off, int K) {
   griddep_wait();
+  griddep_launch();
   const int lane = threadIdx.x & 31;
   const int e = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
   if (e >= E) return;

@@ -111,10 +111,12 @@ def test_fused_pass_rejects_bad_ranges():
         eqb.eqb_margin_hist_lei(z, tau, 2, hist, g, coef, off, 0, T)  # pass 2 without u
 
 
-@pytest.mark.parametrize("T,E,K,M", [(20000, 1024, 8, 64), (20000, 1024, 8, 65), (30000, 256, 8, 300)])
+@pytest.mark.parametrize("T,E,K,M", [(20000, 1024, 8, 64), (20000, 1024, 8, 65), (30000, 256, 8, 300),
+                                     (20000, 128, 8, 4)])
 def test_layer_step_at_and_past_the_coefficient_table(T, E, K, M):
     """M * E = 65,536 runs the fused passes; one microbatch more (or many
-    small ones) runs LEI last.  Both reproduce the oracle."""
+    small ones) runs LEI last.  Both reproduce the oracle, and both give the
+    bits of the separate LEI launch."""
     rng = np.random.default_rng(T + M)
     z = brute.bf16_bits_from_f32(rng.standard_normal((T, E)).astype(np.float32))
     b = (rng.standard_normal(E) * 0.3).astype(np.float32)
@@ -136,6 +138,10 @@ def test_layer_step_at_and_past_the_coefficient_table(T, E, K, M):
     assert np.array_equal(loads.cpu().numpy(), o["loads"])
     assert np.array_equal(bits_f32(bn.cpu().numpy()), bits_f32(o["b_next"]))
     assert within(G.view.cpu().numpy(), g_ref)
+    G2 = torch.from_numpy(g).cuda()
+    eqb.lei_inject_grad(G2, torch.from_numpy(o["loads"]).cuda(), torch.from_numpy(off).cuda(), K, eta, c)
+    torch.cuda.synchronize()
+    assert np.array_equal(bits_f32(G.view.cpu().numpy()), bits_f32(G2.cpu().numpy()))
 
 
 @pytest.mark.parametrize("T", [1, 2, 3, 31, 33, 1025])
