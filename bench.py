@@ -208,9 +208,10 @@ class Step:
         self.off_h = even_offsets(T, self.M)
         self.workspace = torch.zeros(eqb.eqb_layer_workspace_bytes(E), dtype=torch.uint8, device=dev)
         # The one-call step streams LEI inside the two histogram passes when
-        # the [M,E] coefficient table fits its workspace (M * E <= 65,536);
-        # the per-kernel breakdown issues the same kernels through their own
-        # entry points.
+        # the [M,E] coefficient table fits its workspace (M * E <= 65,536),
+        # and each pass's last block runs that pass's selection; the
+        # per-kernel breakdown issues the same work through the separate
+        # entry points (the selections as kernels of their own).
         self.fused = self.M * E <= 65536
         self.coef = torch.empty((self.M, E), dtype=torch.float32, device=dev)
         if workload == "router":
@@ -314,14 +315,14 @@ class Step:
 
     def launches_per_step(self):
         """Kernels of this library launched by one timed one-call step
-        (memsets and torch copies excluded).  Router workload: the projection
-        with routing and the coarse histogram, the LEI coefficient table, two
-        selections (the second with the bias update) and the fine pass
-        carrying LEI: 5.  Otherwise: routing, the coefficient table, two
-        histogram passes carrying the injection, and the two selections (the
-        second with the bias update): 6; without the table, LEI in its own
-        launch instead of the table, still 6."""
-        return 5 if (self.workload == "router" and self.fused) else 6
+        (memsets and torch copies excluded).  Each histogram pass runs its
+        own selection in its last block (the fine pass also the bias update).
+        Router workload: the projection with routing and the coarse
+        histogram, the LEI coefficient table, the pass-1 selection and the
+        fine pass carrying LEI: 4.  Otherwise: routing, the coefficient
+        table and the two histogram passes carrying the injection: 4.
+        Without the table, LEI in its own launch instead: still 4."""
+        return 4
 
     def algorithmic_bytes(self):
         """Bytes the two-pass method must move per step (see the design notes):

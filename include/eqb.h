@@ -204,8 +204,9 @@ eqb_status eqb_margin_hist_lei(const eqb_bf16 *z, const float *tau, int64_t T,
                                void *stream);
 
 /* Bytes of device workspace eqb_layer_step needs for E experts (the two
- * [E,256] histograms, u, rho, q_hat and a 65,536-float LEI coefficient
- * table, each 256-byte aligned; 788,224 bytes for E = 256). */
+ * [E,256] histograms, two block counters, u, rho, q_hat and a 65,536-float
+ * LEI coefficient table, each 256-byte aligned; 788,480 bytes for
+ * E = 256). */
 size_t eqb_layer_workspace_bytes(int32_t E);
 
 /* One layer's whole routing-balance step in one call, in the paper's order:
@@ -215,7 +216,10 @@ size_t eqb_layer_workspace_bytes(int32_t E);
  * to the individual calls above.  When M * E <= 65,536 the LEI coefficients
  * are formed right after routing (lei_coefficients) and the injection is
  * streamed by the two histogram passes, half of the tokens each
- * (eqb_margin_hist_lei); otherwise LEI runs last (lei_inject_grad).
+ * (eqb_margin_hist_lei); otherwise LEI runs last (lei_inject_grad).  Each
+ * histogram pass's selection (eqb_select_quantile; after the fine pass also
+ * eqb_bias_update) runs in the pass's own last block to finish counting,
+ * while the other blocks are still streaming LEI.
  *   z, b, mb_offsets, M, topk_idx (nullable), tau, eta, c: as in
  *             eqb_route_topk / lei_inject_grad;
  *   mb_offsets_host host copy of mb_offsets (nullable; validated when given)
@@ -240,9 +244,9 @@ eqb_status eqb_layer_step(const eqb_bf16 *z, const float *b, int64_t T, int32_t 
  * code that must not stall on or fail at an allocation, can call this
  * instead: it takes the same inputs and outputs but no workspace, and uses a
  * scratch array compiled into the library.
- *   - The scratch is eqb_layer_workspace_bytes(256) = 788,224 bytes: the
- *     step's two histograms, u, rho, q_hat and the 65,536-float LEI
- *     coefficient table, enough for E <= 256; E > 256 returns
+ *   - The scratch is eqb_layer_workspace_bytes(256) = 788,480 bytes: the
+ *     step's two histograms, block counters, u, rho, q_hat and the
+ *     65,536-float LEI coefficient table, enough for E <= 256; E > 256 returns
  *     EQB_ERR_UNSUPPORTED.  Every GPU that loads the library keeps
  *     this array until the process exits.
  *   - The first call on each device looks up the array's device address

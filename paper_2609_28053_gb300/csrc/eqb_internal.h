@@ -67,6 +67,18 @@ struct HistArgs {
   // hist + p*E*256, and pass 2 takes shard p's selected bins from u + p*E.
   const int64_t* shard_off = nullptr;
   int P = 0;
+  // Algorithm 1's selection run by the pass's last block to finish counting
+  // (the one-call step; no shards): *done counts the blocks that finished
+  // (zero before the pass).  Pass 1 selects u, rho at rank r; pass 2 selects
+  // q_hat from u, rho and forms b_next (Eq. 2).  Selection flags go to
+  // sel_err.
+  int32_t* done = nullptr;
+  int64_t r = 0;
+  uint8_t* sel_u = nullptr;
+  int32_t* rho = nullptr;
+  uint16_t* q_hat = nullptr;
+  float* b_next = nullptr;
+  int32_t* sel_err = nullptr;
 };
 
 struct LeiArgs {
@@ -96,11 +108,13 @@ struct GshardArgs {
 constexpr int64_t kLeiCoefCap = 65536;
 
 // The step's scratch, carved from one caller-provided buffer (256-byte
-// aligned pieces): the two [E,256] histograms (adjacent, cleared together
-// before every step), u, rho, q_hat and the [M,E] LEI coefficient table.
+// aligned pieces): the two [E,256] histograms and the passes' two block
+// counters (adjacent, cleared together before every step), u, rho, q_hat and
+// the [M,E] LEI coefficient table.
 struct StepWorkspace {
   int32_t* H;
   int32_t* L;
+  int32_t* done;  // [2]: blocks of pass 1 and of pass 2 done counting
   uint8_t* u;
   int32_t* rho;
   uint16_t* q;
@@ -108,7 +122,7 @@ struct StepWorkspace {
 };
 constexpr size_t carve_round(size_t n) { return (n + 255) / 256 * 256; }
 constexpr size_t step_workspace_bytes(int E) {
-  return 2 * carve_round(static_cast<size_t>(E) * 1024) + carve_round(static_cast<size_t>(E)) +
+  return 2 * carve_round(static_cast<size_t>(E) * 1024) + carve_round(8) + carve_round(static_cast<size_t>(E)) +
          carve_round(4 * static_cast<size_t>(E)) + carve_round(2 * static_cast<size_t>(E)) +
          carve_round(4 * static_cast<size_t>(kLeiCoefCap));
 }

@@ -36,7 +36,7 @@
 // grad_s handed out by a shared counter, so no warp idles while the block
 // has work.  Each pass carries half of the step's tokens, which turns both
 // passes into DRAM-bound ones.
-#include "eqb_device.cuh"
+#include "select_device.cuh"
 
 namespace eqb {
 
@@ -55,6 +55,47 @@ __device__ __forceinline__ void stream_lei(const LeiStream& ls, int E, int* next
   int64_t mlo = 1, mhi = 0;  // token range of microbatch ml (none yet)
   int ml = 0;
   while (lei_warp_next_chunk(ls, E, q0, q1, next, mlo, mhi, ml)) {
+  }
+}
+
+// Algorithm 1's selection in the pass's last block to finish counting (see
+// HistArgs::done), by its nw counting warps (warp wid, lane) with barrier
+// sync(): pass 1 selects u, rho for every expert at rank a.r; pass 2 selects
+// q_hat from u, rho into global memory and a shared copy qs, then forms
+// b_next (Eq. 2).  Each warp loads the counts of three experts at a time
+// (four spill registers of the counting loop); the counts were added by
+// every block's atomics and are read from L2.
+template <int PASS, class Sync>
+__device__ void last_block_select(const HistArgs& a, int nw, int wid, int lane, uint16_t* qs, Sync sync) {
+  constexpr int B = 3;
+  const int E = a.E;
+  for (int e0 = wid; e0 < E; e0 += nw * B) {
+    int4 ca[B], cb[B];
+    int32_t rk[B];
+    uint32_t uk[B];
+#pragma unroll
+    for (int k = 0; k < B; ++k) {
+      const int e = min(e0 + k * nw, E - 1);
+      const int4* h = reinterpret_cast<const int4*>(a.hist + (int64_t)e * 256 + lane * 8);
+      ca[k] = __ldcg(h);
+      cb[k] = __ldcg(h + 1);
+      rk[k] = PASS == 2 ? __ldcg(a.rho + e) : 0;
+      uk[k] = PASS == 2 ? __ldcg(a.sel_u + e) : 0u;
+    }
+#pragma unroll
+    for (int k = 0; k < B; ++k) {
+      const int e = e0 + k * nw;
+      if (e >= E) break;
+      const int64_t cnt[8] = {ca[k].x, ca[k].y, ca[k].z, ca[k].w, cb[k].x, cb[k].y, cb[k].z, cb[k].w};
+      if (PASS == 1)
+        warp_select(cnt, e, 1, a.r, 0u, a.sel_u, a.rho, nullptr, a.sel_err, lane);
+      else
+        warp_select(cnt, e, 2, (int64_t)rk[k], uk[k], a.sel_u, a.rho, a.q_hat, a.sel_err, lane, qs + e);
+    }
+  }
+  if (PASS == 2) {
+    sync();  // every q_hat is in qs
+    block_bias_update<true>(qs, E, a.b_next, nw * 32, sync);
   }
 }
 
@@ -186,6 +227,24 @@ __global__ void __launch_bounds__(1024) hist_kernel(HistArgs a, int64_t tokens_p
     }
     sync_counting();
     cb = ce;
+  }
+  if (PASS != 3 && a.done && !a.shard_off) {
+    // The last block to get here selects.  After the barrier above (every
+    // flush of this block issued), one thread's fence releases the block's
+    // flushes before its count; the last block's fence after its count
+    // orders the other blocks' flushes before its reads.
+    __shared__ int sel_last;
+    if (threadIdx.x == 0) {
+      __threadfence();
+      const bool last = atomicAdd(a.done, 1) == (int)(gridDim.x * gridDim.y) - 1;
+      if (last) __threadfence();
+      sel_last = last;
+    }
+    sync_counting();
+    if (sel_last) {
+      // the bins are clear and no longer used: they hold the q_hat copy
+      last_block_select<PASS>(a, nw, wid, lane, reinterpret_cast<uint16_t*>(bins), sync_counting);
+    }
   }
   if (LEI) stream_lei(ls, E, &lei_next);
 }

@@ -29,6 +29,7 @@ size_t carve_workspace(void* base, int E, StepWorkspace* w) {
   };
   w->H = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 256 * 4));
   w->L = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 256 * 4));
+  w->done = reinterpret_cast<int32_t*>(take(8));
   w->u = take(static_cast<size_t>(E));
   w->rho = reinterpret_cast<int32_t*>(take(static_cast<size_t>(E) * 4));
   w->q = reinterpret_cast<uint16_t*>(take(static_cast<size_t>(E) * 2));
@@ -85,12 +86,41 @@ eqb_status check_step(const eqb_bf16* z, const float* b, int64_t T, int32_t E, i
 }
 
 eqb_status clear(const Workspace& w, int32_t* loads, int32_t E, int32_t M, cudaStream_t s) {
-  // H and L are adjacent in the workspace (each E*1 KiB, a multiple of the
-  // 256-byte carve alignment): one memset clears both.
-  if (cudaMemsetAsync(w.H, 0, 2 * eqb::carve_round(static_cast<size_t>(E) * 1024), s) != cudaSuccess ||
+  // H, L and the block counters are adjacent in the workspace (H and L each
+  // E*1 KiB, a multiple of the 256-byte carve alignment): one memset clears
+  // them.
+  if (cudaMemsetAsync(w.H, 0, 2 * eqb::carve_round(static_cast<size_t>(E) * 1024) + eqb::carve_round(8), s) !=
+          cudaSuccess ||
       cudaMemsetAsync(loads, 0, static_cast<size_t>(M) * E * 4, s) != cudaSuccess)
     return EQB_ERR_CUDA;
   return EQB_OK;
+}
+
+// The two histogram passes of the step, each with its selection run by the
+// pass's last block to finish counting (so neither selection is a launch of
+// its own, and each overlaps the other blocks' LEI streaming): pass 1 counts
+// H and selects u, rho at rank r; pass 2 counts L from u and selects q_hat,
+// then b_next (Eq. 2).
+eqb::HistArgs pass1_args(const Workspace& w, const eqb_bf16* z, const float* tau, int64_t T, int32_t E, int64_t r,
+                         int32_t* err_flag) {
+  eqb::HistArgs h{z, tau, T, E, nullptr, w.H, err_flag};
+  h.done = w.done;
+  h.r = r;
+  h.sel_u = w.u;
+  h.rho = w.rho;
+  h.sel_err = err_flag;
+  return h;
+}
+eqb::HistArgs pass2_args(const Workspace& w, const eqb_bf16* z, const float* tau, int64_t T, int32_t E,
+                         float* b_next, int32_t* err_flag) {
+  eqb::HistArgs h{z, tau, T, E, w.u, w.L, nullptr};
+  h.done = w.done + 1;
+  h.sel_u = w.u;
+  h.rho = w.rho;
+  h.q_hat = w.q;
+  h.b_next = b_next;
+  h.sel_err = err_flag;
+  return h;
 }
 
 // Everything after routing: Algorithm 1's two passes with their selections,
@@ -103,7 +133,8 @@ eqb_status after_routing(const Workspace& w, const eqb_bf16* z, int64_t T, int32
                          const int64_t* mb_offsets, int32_t M, int64_t r, const float* tau,
                          const int32_t* loads, float* b_next, float* grad_s, float eta, float c,
                          int32_t* err_flag, cudaStream_t s) {
-  eqb::HistArgs h1{z, tau, T, E, nullptr, w.H, err_flag};
+  const eqb::HistArgs h1 = pass1_args(w, z, tau, T, E, r, err_flag);
+  const eqb::HistArgs h2 = pass2_args(w, z, tau, T, E, b_next, err_flag);
   if (grad_s && static_cast<int64_t>(M) * E <= eqb::kLeiCoefCap) {
     eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
     if (int rc = eqb::launch_lei_coef(la, w.coef, s)) return st(rc);
@@ -111,17 +142,11 @@ eqb_status after_routing(const Workspace& w, const eqb_bf16* z, int64_t T, int32
     eqb::LeiStream l1{grad_s, w.coef, mb_offsets, M, 0, th};
     eqb::LeiStream l2{grad_s, w.coef, mb_offsets, M, th, T};
     if (int rc = eqb::launch_hist_lei(h1, 1, l1, s)) return st(rc);
-    if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
-    eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};
     if (int rc = eqb::launch_hist_lei(h2, 2, l2, s)) return st(rc);
-    if (int rc = eqb::launch_select_bias(w.L, E, w.u, w.rho, w.q, err_flag, b_next, s)) return st(rc);
     return EQB_OK;
   }
   if (int rc = eqb::launch_hist(h1, 1, s)) return st(rc);
-  if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
-  eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};
   if (int rc = eqb::launch_hist(h2, 2, s)) return st(rc);
-  if (int rc = eqb::launch_select_bias(w.L, E, w.u, w.rho, w.q, err_flag, b_next, s)) return st(rc);
   if (grad_s) {
     eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
     if (int rc = eqb::launch_lei(la, s)) return st(rc);
@@ -130,9 +155,9 @@ eqb_status after_routing(const Workspace& w, const eqb_bf16* z, int64_t T, int32
 }
 
 // Everything after routing when the coarse histogram H was already counted
-// (the router projection's epilogue): selection, the fine pass, selection
-// and the bias update, with LEI streamed entirely by the fine pass when the
-// [M,E] coefficient table fits the workspace, else run last.
+// (the router projection's epilogue): selection, the fine pass with its
+// selection and the bias update, with LEI streamed entirely by the fine pass
+// when the [M,E] coefficient table fits the workspace, else run last.
 eqb_status after_coarse(const Workspace& w, const eqb_bf16* z, int64_t T, int32_t E, int32_t K,
                         const int64_t* mb_offsets, int32_t M, int64_t r, const float* tau, const int32_t* loads,
                         float* b_next, float* grad_s, float eta, float c, int32_t* err_flag, cudaStream_t s) {
@@ -142,17 +167,16 @@ eqb_status after_coarse(const Workspace& w, const eqb_bf16* z, int64_t T, int32_
     if (int rc = eqb::launch_lei_coef(la, w.coef, s)) return st(rc);
   }
   if (int rc = eqb::launch_select(w.H, E, 1, r, w.u, w.rho, nullptr, err_flag, s)) return st(rc);
-  eqb::HistArgs h2{z, tau, T, E, w.u, w.L, nullptr};
+  const eqb::HistArgs h2 = pass2_args(w, z, tau, T, E, b_next, err_flag);
   if (lei) {
     eqb::LeiStream l2{grad_s, w.coef, mb_offsets, M, 0, T};
     if (int rc = eqb::launch_hist_lei(h2, 2, l2, s)) return st(rc);
   } else {
     if (int rc = eqb::launch_hist(h2, 2, s)) return st(rc);
-  }
-  if (int rc = eqb::launch_select_bias(w.L, E, w.u, w.rho, w.q, err_flag, b_next, s)) return st(rc);
-  if (grad_s && !lei) {
-    eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
-    if (int rc = eqb::launch_lei(la, s)) return st(rc);
+    if (grad_s) {
+      eqb::LeiArgs la{grad_s, loads, mb_offsets, M, 0, T, E, K, eta, c};
+      if (int rc = eqb::launch_lei(la, s)) return st(rc);
+    }
   }
   return EQB_OK;
 }

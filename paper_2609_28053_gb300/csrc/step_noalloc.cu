@@ -9,9 +9,9 @@
 // [E,256] histograms, u, rho and q_hat) lives here.
 //
 // The scratch is one file-scope device array sized for the largest supported
-// E (256 experts): eqb_layer_workspace_bytes(256) = 788,224 bytes (the two
-// [256,256] histograms, u, rho, q_hat and the 65,536-float LEI coefficient
-// table).  Every GPU that loads this library
+// E (256 experts): eqb_layer_workspace_bytes(256) = 788,480 bytes (the two
+// [256,256] histograms, two block counters, u, rho, q_hat and the
+// 65,536-float LEI coefficient table).  Every GPU that loads this library
 // holds it until the process exits.  Host code cannot use the array's name as a
 // device address, so the first call on each device, with that device
 // current, looks the address up once with cudaGetSymbolAddress; make that

@@ -207,9 +207,9 @@ def test_layer_step_workspace_size(lib):
     assert lib.eqb_layer_workspace_bytes(256) % 256 == 0
     assert lib.eqb_layer_workspace_bytes(0) == 0
     # the size the header and the allocation-free entry point state
-    assert lib.eqb_layer_workspace_bytes(256) == 788224
+    assert lib.eqb_layer_workspace_bytes(256) == 788480
     src = open(HEADER).read()
-    assert "788,224 bytes" in src
+    assert "788,480 bytes" in src
 
 
 def test_layer_step_rejects(lib):
