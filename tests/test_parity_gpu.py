@@ -485,3 +485,48 @@ def test_layer_step_matches_oracle(T, E, K, M):
     assert np.array_equal(bits_f32(bn.view.cpu().numpy()), bits_f32(o["b_next"]))
     got = G.view.cpu().numpy().astype(np.float64)
     assert np.all(np.abs(got - g_ref) <= LEI_ATOL + LEI_RTOL * np.abs(g_ref))
+
+
+def test_layer_step_unreachable_rank_sets_flag():
+    """A target rank above T cannot be reached: the selection that the
+    coarse pass's last block runs inside the one-call step raises
+    EQB_ERR_RANK, as the separate selection does."""
+    T, E, K = 3000, 64, 8
+    z, b = rand_case(T, E, seed=11)
+    off = np.array([0, T], np.int64)
+    loads = torch.zeros((1, E), dtype=torch.int32, device="cuda")
+    bn = torch.zeros(E, dtype=torch.float32, device="cuda")
+    ws = torch.zeros(eqb.eqb_layer_workspace_bytes(E), dtype=torch.uint8, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    eqb.eqb_layer_step(to_dev_bf16(z), torch.from_numpy(b).cuda(), K, torch.from_numpy(off).cuda(), loads, bn,
+                       ws, r=T + 1, mb_offsets_host=off, err_flag=err)
+    torch.cuda.synchronize()
+    assert err.item() == 5
+
+
+@pytest.mark.parametrize("T,E,K,M", [(200000, 256, 8, 8), (3000, 64, 8, 3)])
+def test_layer_step_reuses_its_workspace(T, E, K, M):
+    """Two steps on different inputs through one workspace: the second
+    reproduces the oracle on its own inputs (the passes' block counters and
+    histograms are cleared for every step, so each pass's last block
+    selects again)."""
+    ws = torch.full((eqb.eqb_layer_workspace_bytes(E),), 0x5a, dtype=torch.uint8, device="cuda")
+    off = ragged_offsets(T, M, seed=M)
+    offd = torch.from_numpy(off).cuda()
+    for seed in (1, 2):
+        z, b = rand_case(T, E, seed=T + seed)
+        g = (np.random.default_rng(seed).standard_normal((T, E)) * 0.1).astype(np.float32)
+        o = oracle_forward(z, b, K, off)
+        g_ref, _ = oracle.lei(g, o["loads"], off, K, 0.5, 1.0)
+        loads = torch.zeros((M, E), dtype=torch.int32, device="cuda")
+        bn = torch.zeros(E, dtype=torch.float32, device="cuda")
+        G = torch.from_numpy(g).cuda()
+        err = torch.zeros(1, dtype=torch.int32, device="cuda")
+        eqb.eqb_layer_step(to_dev_bf16(z), torch.from_numpy(b).cuda(), K, offd, loads, bn, ws, grad_s=G, eta=0.5,
+                           c=1.0, mb_offsets_host=off, err_flag=err)
+        torch.cuda.synchronize()
+        assert err.item() == 0
+        assert np.array_equal(loads.cpu().numpy(), o["loads"])
+        assert np.array_equal(bits_f32(bn.cpu().numpy()), bits_f32(o["b_next"]))
+        got = G.cpu().numpy().astype(np.float64)
+        assert np.all(np.abs(got - g_ref) <= LEI_ATOL + LEI_RTOL * np.abs(g_ref))
