@@ -148,11 +148,6 @@ int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, i
 int launch_select_sharded(const int32_t* hist, int E, int pass, const int64_t* shard_off, int P, int K,
                           uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err, cudaStream_t s);
 int launch_bias_update(const uint16_t* q_hat, int E, float* b_next, cudaStream_t s);
-// The pass-2 selection of every expert and the Eq. (2) bias update in one
-// single-block launch (the same results as launch_select(pass 2) followed by
-// launch_bias_update).
-int launch_select_bias(const int32_t* hist, int E, const uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err,
-                       float* b_next, cudaStream_t s);
 int launch_lei(const LeiArgs& a, cudaStream_t s);
 // The [M,E] fp32 table of Eq. (norm) coefficients, row l for microbatch l
 // (bit-identical to the coefficients launch_lei forms).

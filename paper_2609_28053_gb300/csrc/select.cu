@@ -19,8 +19,6 @@ namespace eqb {
 
 namespace {
 
-constexpr int kSelectBiasMaxE = 1024;  // experts of one select_bias_kernel block
-
 __global__ void __launch_bounds__(256) select_kernel(const int32_t* __restrict__ hist, int E, int pass,
                                                      int64_t r, uint8_t* __restrict__ u,
                                                      int32_t* __restrict__ rho,
@@ -62,46 +60,6 @@ __global__ void bias_update_kernel(const uint16_t* __restrict__ q_hat, int E, fl
   block_bias_update<false>(q_hat, E, b_next, blockDim.x, [] { __syncthreads(); });
 }
 
-// Algorithm 1 steps 5-6 and Eq. (2) in one block: the pass-2 selection of
-// every expert (each warp loads the counts, rho and u of 4 experts before it
-// scans them, so a batch costs one L2 round trip), then the bias update from
-// the block's shared copy of q_hat.  Same results as select_kernel (pass 2)
-// followed by bias_update_kernel.  E <= kSelectBiasMaxE.
-__global__ void __launch_bounds__(1024) select_bias_kernel(const int32_t* __restrict__ hist, int E,
-                                                           const uint8_t* __restrict__ u,
-                                                           int32_t* __restrict__ rho,
-                                                           uint16_t* __restrict__ q_hat, int32_t* err,
-                                                           float* __restrict__ b_next) {
-  constexpr int B = 4;
-  __shared__ uint16_t qs[kSelectBiasMaxE];
-  griddep_wait();
-  const int lane = threadIdx.x & 31, wid = threadIdx.x >> 5, nw = blockDim.x >> 5;
-  for (int e0 = wid; e0 < E; e0 += nw * B) {
-    int4 ca[B], cb[B];
-    int32_t rk[B];
-    uint32_t uk = 0u;  // u of the batch, one byte per expert
-#pragma unroll
-    for (int k = 0; k < B; ++k) {
-      const int e = min(e0 + k * nw, E - 1);
-      const int32_t* h = hist + (int64_t)e * 256 + lane * 8;
-      ca[k] = __ldg(reinterpret_cast<const int4*>(h));
-      cb[k] = __ldg(reinterpret_cast<const int4*>(h + 4));
-      rk[k] = __ldcg(rho + e);
-      uk |= static_cast<uint32_t>(__ldcg(u + e)) << (8 * k);
-    }
-#pragma unroll
-    for (int k = 0; k < B; ++k) {
-      const int e = e0 + k * nw;
-      const int64_t cnt[8] = {ca[k].x, ca[k].y, ca[k].z, ca[k].w, cb[k].x, cb[k].y, cb[k].z, cb[k].w};
-      if (e < E)
-        warp_select(cnt, e, 2, (int64_t)rk[k], (uk >> (8 * k)) & 0xffu, const_cast<uint8_t*>(u), rho, q_hat, err,
-                    lane, qs + e);
-    }
-  }
-  __syncthreads();  // every q_hat is written
-  block_bias_update<true>(qs, E, b_next, blockDim.x, [] { __syncthreads(); });
-}
-
 }  // namespace
 
 int launch_select(const int32_t* hist, int E, int pass, int64_t r, uint8_t* u, int32_t* rho,
@@ -120,15 +78,6 @@ int launch_select_sharded(const int32_t* hist, int E, int pass, const int64_t* s
   dim3 grid((E + wpb - 1) / wpb, P);
   return launch_dependent(select_kernel, grid, dim3(wpb * 32), 0, s, hist, E, pass, (int64_t)0, u, rho, q_hat, err,
                           shard_off, K) == cudaSuccess
-             ? kOk
-             : kErrCuda;
-}
-
-int launch_select_bias(const int32_t* hist, int E, const uint8_t* u, int32_t* rho, uint16_t* q_hat, int32_t* err,
-                       float* b_next, cudaStream_t s) {
-  if (E > kSelectBiasMaxE) return kErrUnsupported;
-  return launch_dependent(select_bias_kernel, dim3(1), dim3(1024), 0, s, hist, E, u, rho, q_hat, err, b_next) ==
-                 cudaSuccess
              ? kOk
              : kErrCuda;
 }
