@@ -321,7 +321,9 @@ class Step:
         histogram, the LEI coefficient table, the pass-1 selection and the
         fine pass carrying LEI: 4.  Otherwise: routing, the coefficient
         table and the two histogram passes carrying the injection: 4.
-        Without the table, LEI in its own launch instead: still 4."""
+        Without the table, LEI in its own launch instead: still 4.  (With
+        several ranks the histograms are summed between the passes, so the
+        step runs as the separate calls of `names`, one kernel each.)"""
         return 4
 
     def algorithmic_bytes(self):
@@ -882,7 +884,7 @@ def main():
                                   "timed region)" if args.workload in SMALL_WORKLOADS else
                                   "inputs larger than L2 (at least 1 GiB each); no flush"),
                            "parallelism": f"dp{world}"},
-                "gpu_launches": step.launches_per_step() * args.steps,
+                "gpu_launches": (step.launches_per_step() if one_call else len(step.names)) * args.steps,
                 "schedule": ("one eqb_layer_step call per step" if one_call
                              else "per-pass calls, histograms all-reduced"),
                 "roofline": roofline,
